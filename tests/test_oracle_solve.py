@@ -1,0 +1,93 @@
+"""Pins for the oracle's right-hand sides, operator and CG (§3.1.2-§3.1.3, Eq. 4-5).
+
+* Y = B^T W^{1/2} Q is compared with the dense incidence product, checked to lie in range(L)
+  (1^T Y = 0 on every connected component) and checked statistically against E[Y Y^T] = L.
+* L_eps X is compared with the dense (B^T W B + eps I) X.
+* CG is compared with a direct dense solve (the paper's ERC-JL) and its true residual with tau.
+"""
+import numpy as np
+import pytest
+import scipy.sparse.csgraph as csg
+
+from oracle import dense as D
+from oracle import erc_oracle as O
+from paper_2609_27209_gb300 import synth
+
+
+def _graph(seed=0, n=60, extra=150):
+    n, src, dst, w = synth.random_connected(n, extra, seed)
+    return O.build_laplacian(n, src, dst, w)
+
+
+def test_rhs_equals_dense_incidence_product():
+    g = _graph(1)
+    K, c0, kc = 300, 40, 200
+    Y = O.jl_rhs(g, 99, K, c0, kc, edge_block=37)
+    B = D.dense_incidence(g["n"], g["eu"], g["ev"])
+    Q = O.jl_q(99, K, np.arange(g["m"]), c0, kc)
+    ref = B.T @ (np.sqrt(g["ew"].astype(np.float64))[:, None] * Q)
+    np.testing.assert_allclose(Y, ref, rtol=0, atol=1e-13)
+
+
+def test_rhs_lies_in_range_of_laplacian_per_component():
+    n, src, dst, w = synth.random_multigraph(80, 70, 5, self_loops=True)
+    g = O.build_laplacian(n, src, dst, w)
+    ncomp, lab = csg.connected_components(O.adjacency(g), directed=False)
+    assert ncomp > 1
+    Y = O.jl_rhs(g, 3, 64, 0, 64)
+    for c in range(ncomp):
+        np.testing.assert_allclose(Y[lab == c].sum(axis=0), 0.0, atol=1e-12)
+
+
+def test_rhs_second_moment_is_laplacian():
+    g = _graph(2, n=12, extra=20)
+    K = 16384
+    Y = O.jl_rhs(g, 11, K, 0, K)
+    L = D.dense_laplacian(g["n"], g["eu"], g["ev"], g["ew"])
+    M = Y @ Y.T
+    d = np.diag(L)
+    bound = 6.0 * np.sqrt(2.0 * np.outer(d, d) / K)
+    assert np.all(np.abs(M - L) <= bound + 1e-12)
+
+
+def test_matvec_equals_dense_regularized_laplacian():
+    g = _graph(3)
+    rng = np.random.default_rng(0)
+    X = rng.standard_normal((g["n"], 7))
+    L = D.dense_laplacian(g["n"], g["eu"], g["ev"], g["ew"])
+    np.testing.assert_allclose(O.laplacian_matvec(g, 1e-3, X),
+                               (L + 1e-3 * np.eye(g["n"])) @ X, rtol=0, atol=1e-11)
+
+
+@pytest.mark.parametrize("eps", [1e-3, 1e-1])
+def test_cg_matches_direct_solve(eps):
+    g = _graph(4, n=150, extra=300)
+    Y = O.jl_rhs(g, 5, 32, 0, 32)
+    X, iters, relres, ok = O.batched_cg(g, eps, Y, 1e-11)
+    assert ok
+    Z = D.jl_dense_solve(D.dense_laplacian(g["n"], g["eu"], g["ev"], g["ew"]), eps, Y)
+    np.testing.assert_allclose(X, Z, rtol=0, atol=1e-7 * np.abs(Z).max())
+    assert np.all(relres <= 1e-11 * 1.01)
+    assert np.all(iters > 0) and np.all(iters <= 3 * g["n"])
+
+
+def test_cg_zero_column_and_max_iter():
+    g = _graph(5)
+    Y = O.jl_rhs(g, 6, 8, 0, 8)
+    Y[:, 3] = 0.0
+    X, iters, relres, ok = O.batched_cg(g, 1e-3, Y, 1e-8)
+    assert ok and iters[3] == 0 and np.all(X[:, 3] == 0) and relres[3] == 0
+    X, iters, relres, ok = O.batched_cg(g, 1e-3, Y, 1e-8, max_iter=2)
+    assert not ok and np.all(iters[np.arange(8) != 3] == 2)
+
+
+def test_cg_stops_columns_independently():
+    """Each column's iterate equals a single-column solve of that column alone."""
+    g = _graph(6, n=100, extra=200)
+    Y = O.jl_rhs(g, 8, 16, 0, 16)
+    Y[:, 0] *= 1e-3  # differently scaled columns still stop on their own relative residual
+    X, iters, _, _ = O.batched_cg(g, 1e-3, Y, 1e-6)
+    for c in [0, 5, 15]:
+        x1, it1, _, _ = O.batched_cg(g, 1e-3, Y[:, c:c + 1], 1e-6)
+        assert it1[0] == iters[c]
+        np.testing.assert_allclose(X[:, c], x1[:, 0], rtol=1e-12, atol=1e-15)
