@@ -1,0 +1,204 @@
+/*
+ * erc.h -- C ABI of liberc.so: ERC-LG (effective-resistance curvature of every edge of a large graph)
+ * on one NVIDIA GB300 GPU (sm_103a).
+ *
+ * Method: "Scalable Subgraph Sampling via Resistance Curvature" (arxiv 2609.27209), §3.
+ *   L = D - A = B^T W B (§3.1.1); Y = B^T W^{1/2} Q with Q_ec uniform on {+-1/sqrt(K)} (§3.1.2);
+ *   column-wise CG on L_eps Z = Y, L_eps = L + eps I (Eq. 5, §3.1.3, Algorithm 1);
+ *   R_uv = ||Z_u - Z_v||^2 accumulated over column batches (Eq. 6, Algorithm 1);
+ *   p_u = 1 - 1/2 sum_v w_uv R_uv, kappa_uv = 2 (p_u + p_v) / R_uv (Eq. 2);
+ *   node / edge sampling probabilities (Eq. 7, Eq. 8, §3.2).
+ *
+ * Conventions for every call
+ *   - Returns an erc_status; erc_last_error() gives a message for the last failure on the calling
+ *     host thread.
+ *   - Array arguments are DEVICE pointers owned by the caller unless marked "host".  The library
+ *     never frees or keeps caller memory and performs no device allocation: scratch space comes
+ *     from the caller through the matching *_workspace_size() query (16-byte alignment or better;
+ *     the library aligns sub-buffers itself).
+ *   - Work is ordered on the caller's stream `s` (a cudaStream_t; NULL = legacy default stream)
+ *     and is asynchronous, except where a host-visible result is returned (m_out, the CG status):
+ *     those calls synchronise `s` before returning.
+ *   - Node ids are int32 in [0, n); CSR offsets are int64.  Column blocks (Y, X) are row-major
+ *     n x ld float32 with ld >= kc, ld a multiple of 4 and the base 16-byte aligned; only the
+ *     first kc columns of a row carry data.
+ *   - Precision: float32 storage and arithmetic; dot products and per-column CG scalars are
+ *     accumulated in a float32 pair (about 44 significant bits) and finished in float64.
+ */
+#ifndef ERC_H
+#define ERC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void* erc_stream; /* cudaStream_t */
+
+typedef enum erc_status {
+  ERC_OK = 0,
+  ERC_ERR_INVALID_ARG = 1,   /* bad size, pointer, alignment, node id or weight */
+  ERC_ERR_CUDA = 2,          /* a CUDA runtime call failed (message has the CUDA error) */
+  ERC_ERR_CAPACITY = 3,      /* workspace too small, or a size beyond the library's limits */
+  ERC_ERR_NOT_CONVERGED = 4, /* some CG column reached max_iter; results are still written */
+  ERC_ERR_NUMERIC = 5,       /* a non-finite or non-positive CG scalar was met */
+  ERC_ERR_TIMEOUT = 6        /* a bounded device-side wait ran out */
+} erc_status;
+
+enum { ERC_DUP_SUM = 0, ERC_DUP_FIRST = 1 };
+
+/* Non-owning view of a graph built by erc_build_laplacian (all pointers device, read-only). */
+typedef struct erc_graph {
+  int32_t n;              /* nodes */
+  int64_t m;              /* undirected edges; the CSR holds 2m slots */
+  const int64_t* row_ptr; /* [n+1] CSR offsets of the symmetric adjacency A */
+  const int32_t* col;     /* [2m] neighbour ids, strictly ascending within a row */
+  const float* val;       /* [2m] edge weights w_uv, or NULL when every weight is 1 */
+  const float* deg;       /* [n] weighted degree sum_v w_uv (float64 sum, rounded once) */
+  const int32_t* csr_eid; /* [2m] canonical edge id of each CSR slot */
+  const int32_t* eu;      /* [m] canonical edges: eu[e] < ev[e], lexicographic order */
+  const int32_t* ev;      /* [m] */
+  const float* ew;        /* [m] weight of edge e, or NULL when every weight is 1 */
+} erc_graph;
+
+/* Parameters of a whole ERC-LG run (Algorithm 1 + §3.2). */
+typedef struct erc_params {
+  uint64_t seed;      /* Philox key of Q */
+  int32_t K;          /* projection dimension (§3.1.2) */
+  int32_t kc;         /* columns per streamed batch ("b" in Algorithm 1), 1..1024 */
+  float eps;          /* regularisation eps > 0 (Eq. 5) */
+  float tol;          /* CG relative residual tolerance tau (Algorithm 1) */
+  int32_t max_iter;   /* CG iteration cap per column */
+  float eta;          /* eta > 0 of Eq. 7 */
+  int32_t dup_policy; /* ERC_DUP_SUM or ERC_DUP_FIRST */
+} erc_params;
+
+const char* erc_version(void);
+const char* erc_last_error(void);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_build_laplacian -- the simple undirected graph behind L = D - A = B^T W B (§3.1.1).
+ *
+ * In : n nodes; src, dst [m_in] int32 endpoints (any order/orientation); w [m_in] float32 weights
+ *      (> 0, finite) or NULL for unit weights; dup_policy: repeated (u,v) pairs (either
+ *      orientation) are merged by summing their weights in float64 in input order and rounding
+ *      once (ERC_DUP_SUM) or by keeping the first weight (ERC_DUP_FIRST).  Self-loops are dropped
+ *      (they contribute nothing to B^T W B).
+ * Out: row_ptr [n+1], col [2 m_in], val [2 m_in] (may be NULL only when w is NULL), deg [n],
+ *      csr_eid [2 m_in], eu, ev [m_in], ew [m_in] (may be NULL); capacities in brackets, the first
+ *      2m / m entries are written; m_out (host) receives m.  Edge ids e = 0..m-1 number the
+ *      canonical pairs (eu < ev) in lexicographic order.  Deterministic (bit-identical reruns).
+ * Errors: INVALID_ARG for n < 1, m_in < 0 or > 2^30, an id outside [0, n), a weight <= 0 or
+ *      non-finite; CAPACITY if ws_bytes < erc_build_laplacian_workspace_size(n, m_in).
+ * Synchronises s.
+ * ------------------------------------------------------------------------------------------- */
+size_t erc_build_laplacian_workspace_size(int32_t n, int64_t m_in);
+erc_status erc_build_laplacian(int32_t n, const int32_t* src, const int32_t* dst, const float* w,
+                               int64_t m_in, int32_t dup_policy, int64_t* row_ptr, int32_t* col,
+                               float* val, float* deg, int32_t* csr_eid, int32_t* eu, int32_t* ev,
+                               float* ew, int64_t* m_out, void* ws, size_t ws_bytes, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_jl_rhs -- Y[:, 0:kc] = (B^T W^{1/2} Q)[:, c0:c0+kc]  (§3.1.2; Algorithm 1 "form Y").
+ *
+ * Row e of B is e_u - e_v for the canonical edge (u = eu[e] < v = ev[e]).  Q is never stored: its
+ * entry (e, c) is +1/sqrt(K) when a Philox4x32-10 bit is 0 and -1/sqrt(K) when it is 1, the bit
+ * being bit (c mod 32) of word ((c div 32) mod 4) of Philox4x32-10 with key (seed lo, seed hi) and
+ * counter (c div 128, 0, e lo, e hi).  K is the total projection dimension, so a column's values
+ * do not depend on the batch it is produced in.  Requires c0 % 4 == 0, 0 < kc, c0 + kc <= K.
+ * Row u is summed in CSR order (deterministic).  Columns kc..ld-1 are set to 0.
+ * ------------------------------------------------------------------------------------------- */
+erc_status erc_jl_rhs(const erc_graph* g, uint64_t seed, int32_t K, int32_t c0, int32_t kc,
+                      float* Y, int32_t ld, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_batched_cg -- solve L_eps X = Y column by column with CG (Eq. 5, §3.1.3, Algorithm 1).
+ *
+ * Every column c < kc runs Hestenes-Stiefel CG from x = 0 independently of the others and stops
+ * once its recursively updated residual satisfies ||r||_2 <= tol ||y||_2, or after max_iter
+ * iterations.  L_eps p is applied as eps p_u + sum_v w_uv (p_u - p_v).
+ * Out: X [n x ld] (columns kc..ld-1 set to 0); iters [kc] int32 (device) iterations per column;
+ *      relres [kc] float (device) true relative residual ||y - L_eps x|| / ||y|| of the returned x.
+ * Errors: NOT_CONVERGED if any column stopped at max_iter; NUMERIC if p^T L_eps p <= 0 or a
+ *      non-finite scalar appeared (that column is frozen); CAPACITY if ws is too small.
+ * Synchronises s (it reads the convergence status).
+ * ------------------------------------------------------------------------------------------- */
+size_t erc_batched_cg_workspace_size(int32_t n, int32_t ld);
+erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* X, int32_t ld,
+                          int32_t kc, float tol, int32_t max_iter, int32_t* iters, float* relres,
+                          void* ws, size_t ws_bytes, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_edge_resistance -- R_acc[e] += sum_{c < kc} (X[eu[e], c] - X[ev[e], c])^2   (Eq. 6).
+ *
+ * Called once per column batch on the batch's solution, so R_acc (float32 [m], zeroed by the
+ * caller before the first batch) ends as the JL estimate over all K columns without the n x K
+ * embedding ever being held (Algorithm 1's streamed accumulation).
+ * ------------------------------------------------------------------------------------------- */
+erc_status erc_edge_resistance(const erc_graph* g, const float* X, int32_t ld, int32_t kc,
+                               float* R_acc, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_curvature -- Eq. 2: p_u = 1 - 1/2 sum_{v in N(u)} w_uv R_uv (float64 row sums),
+ *                  kappa_e = 2 (p_u + p_v) / R_e for e = (u, v).
+ * In: R [m].  Out: p_node [n], kappa [m].  R_e = 0 gives an IEEE infinity / NaN.
+ * ------------------------------------------------------------------------------------------- */
+erc_status erc_curvature(const erc_graph* g, const float* R, float* p_node, float* kappa,
+                         erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_sampling_probs -- §3.2.
+ *   node: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta)  (Eq. 7);
+ *         prob_node = q / sum q, or, when every q_u is 0, uniform over the nodes with an edge.
+ *   edge: q_e = sqrt(max(-kappa_e + 2 kappa_max, 0)) + 1 (Eq. 8); prob_edge = q / sum q over the
+ *         m canonical edges.
+ * Out: prob_node [n], prob_edge [m].  Sums are float64 in a fixed order (deterministic).
+ * ------------------------------------------------------------------------------------------- */
+size_t erc_sampling_probs_workspace_size(int32_t n, int64_t m);
+erc_status erc_sampling_probs(const erc_graph* g, const float* kappa, float eta, float* prob_node,
+                              float* prob_edge, void* ws, size_t ws_bytes, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_laplacian_apply -- AP = L_eps P for an n x ld block (the CG operator of Eq. 5), and, when
+ * pAp is not NULL, pAp[c] = sum_u P[u,c] AP[u,c] as float64 (device [kc]).  Exposed for testing
+ * and benchmarking the operator alone.
+ * ------------------------------------------------------------------------------------------- */
+size_t erc_laplacian_apply_workspace_size(int32_t n, int32_t ld);
+erc_status erc_laplacian_apply(const erc_graph* g, float eps, const float* P, float* AP,
+                               int32_t ld, int32_t kc, double* pAp, void* ws, size_t ws_bytes,
+                               erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_philox_signs -- the sign bits of Q[e, c] for e in [e0, e1), c in [c0, c1) (see erc_jl_rhs),
+ * written to out_bits (device, row-major (e1-e0) x (c1-c0), one uint32 0/1 per entry).
+ * ------------------------------------------------------------------------------------------- */
+erc_status erc_philox_signs(uint64_t seed, int64_t e0, int64_t e1, int32_t c0, int32_t c1,
+                            uint32_t* out_bits, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
+ * erc_run -- the whole path: erc_build_laplacian, then for c0 = 0, kc, 2kc, ... < K:
+ * erc_jl_rhs -> erc_batched_cg -> erc_edge_resistance (Algorithm 1), then erc_curvature and
+ * erc_sampling_probs.  Inputs as erc_build_laplacian; outputs (device, capacity m_in for the edge
+ * arrays): eu, ev [m], R [m], p_node [n], kappa [m], prob_node [n], prob_edge [m], iters [K],
+ * relres [K]; m_out (host).  NOT_CONVERGED is reported after all batches are done.
+ * erc_run_host is the same with src, dst, w and every output in HOST memory (pinned memory
+ * makes the copies asynchronous); the copies run on s inside the call.
+ * ------------------------------------------------------------------------------------------- */
+size_t erc_run_workspace_size(int32_t n, int64_t m_in, int32_t kc);
+erc_status erc_run(const erc_params* prm, int32_t n, const int32_t* src, const int32_t* dst,
+                   const float* w, int64_t m_in, int64_t* m_out, int32_t* eu, int32_t* ev,
+                   float* R, float* p_node, float* kappa, float* prob_node, float* prob_edge,
+                   int32_t* iters, float* relres, void* ws, size_t ws_bytes, erc_stream s);
+size_t erc_run_host_workspace_size(int32_t n, int64_t m_in, int32_t kc, int32_t K);
+erc_status erc_run_host(const erc_params* prm, int32_t n, const int32_t* src, const int32_t* dst,
+                        const float* w, int64_t m_in, int64_t* m_out, int32_t* eu, int32_t* ev,
+                        float* R, float* p_node, float* kappa, float* prob_node,
+                        float* prob_edge, int32_t* iters, float* relres, void* ws,
+                        size_t ws_bytes, erc_stream s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ERC_H */

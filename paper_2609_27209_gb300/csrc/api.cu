@@ -1,0 +1,257 @@
+// api.cu -- error reporting, graph checks and the whole-path drivers erc_run / erc_run_host
+// (Algorithm 1 followed by §3.2), which stream the K projection columns in batches of kc so the
+// n x K embedding is never held.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "erc_internal.cuh"
+
+namespace erc {
+
+namespace {
+thread_local char g_err[512] = "";
+}
+
+erc_status set_error(erc_status code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof g_err, fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+void clear_error() { g_err[0] = '\0'; }
+
+int sm_count() {
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (!cache[dev]) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
+      v = 148;
+    cache[dev] = v;
+  }
+  return cache[dev];
+}
+
+erc_status check_graph(const erc_graph* g) {
+  ERC_REQUIRE(g, "graph is null");
+  ERC_REQUIRE(g->n >= 1, "graph has n < 1");
+  ERC_REQUIRE(g->m >= 0 && g->m < (int64_t(1) << 31), "graph m out of range");
+  ERC_REQUIRE(g->row_ptr, "graph row_ptr is null");
+  ERC_REQUIRE(g->m == 0 || (g->col && g->csr_eid && g->eu && g->ev), "graph arrays are null");
+  return ERC_OK;
+}
+
+namespace {
+
+__global__ void k_all_unit(const float* __restrict__ w, int64_t m, int* __restrict__ nonunit) {
+  int bad = 0;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < m;
+       e += (int64_t)gridDim.x * blockDim.x)
+    bad |= (w[e] != 1.f);
+  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(nonunit, 1);
+}
+
+struct RunPlan {
+  int64_t* row_ptr;
+  int32_t *col, *csr_eid;
+  float *val, *deg, *ew;
+  float *Y, *X;
+  int* flag;
+  void* cg_ws;
+  size_t cg_bytes;
+  void* aux_ws;  // build workspace, later the sampling workspace
+  size_t aux_bytes;
+};
+
+inline int32_t ld_for(int32_t kc) { return (kc + 3) & ~3; }
+
+void plan_run(Arena& a, RunPlan& p, int32_t n, int64_t m_in, int32_t kc) {
+  const int32_t ld = ld_for(kc);
+  p.row_ptr = a.take<int64_t>((size_t)n + 1);
+  p.col = a.take<int32_t>(2 * m_in);
+  p.csr_eid = a.take<int32_t>(2 * m_in);
+  p.val = a.take<float>(2 * m_in);
+  p.deg = a.take<float>(n);
+  p.ew = a.take<float>(m_in);
+  p.Y = a.take<float>((size_t)n * ld);
+  p.X = a.take<float>((size_t)n * ld);
+  p.flag = a.take<int>(4);
+  p.cg_bytes = erc_batched_cg_workspace_size(n, ld);
+  p.cg_ws = a.take<char>(p.cg_bytes);
+  const size_t b1 = erc_build_laplacian_workspace_size(n, m_in);
+  const size_t b2 = erc_sampling_probs_workspace_size(n, m_in);
+  p.aux_bytes = b1 > b2 ? b1 : b2;
+  p.aux_ws = a.take<char>(p.aux_bytes);
+}
+
+erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, const int32_t* dst,
+                      const float* w, int64_t m_in, int64_t* m_out, int32_t* eu, int32_t* ev,
+                      float* R, float* p_node, float* kappa, float* prob_node, float* prob_edge,
+                      int32_t* iters, float* relres, const RunPlan& p, cudaStream_t s) {
+  const int32_t ld = ld_for(prm->kc);
+  int64_t m = 0;
+  ERC_TRY(erc_build_laplacian(n, src, dst, w, m_in, prm->dup_policy, p.row_ptr, p.col, p.val,
+                              p.deg, p.csr_eid, eu, ev, p.ew, &m, p.aux_ws, p.aux_bytes,
+                              reinterpret_cast<erc_stream>(s)));
+  *m_out = m;
+  // an unweighted input whose duplicates did not merge keeps unit weights: drop the weight
+  // arrays so the gathers read indices only
+  int nonunit = 1;
+  if (!w && m > 0) {
+    ERC_CUDA(cudaMemsetAsync(p.flag, 0, sizeof(int), s));
+    k_all_unit<<<grid_for(m, 256), 256, 0, s>>>(p.ew, m, p.flag);
+    ERC_CUDA(cudaGetLastError());
+    ERC_CUDA(cudaMemcpyAsync(&nonunit, p.flag, sizeof(int), cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaStreamSynchronize(s));
+  }
+  erc_graph g{n, m, p.row_ptr, p.col, nonunit ? p.val : nullptr, p.deg, p.csr_eid,
+              eu, ev, nonunit ? p.ew : nullptr};
+  if (m > 0) ERC_CUDA(cudaMemsetAsync(R, 0, (size_t)m * sizeof(float), s));
+  erc_status worst = ERC_OK;
+  for (int32_t c0 = 0; c0 < prm->K; c0 += prm->kc) {
+    const int32_t k = prm->kc < prm->K - c0 ? prm->kc : prm->K - c0;
+    ERC_TRY(erc_jl_rhs(&g, prm->seed, prm->K, c0, k, p.Y, ld, reinterpret_cast<erc_stream>(s)));
+    erc_status st = erc_batched_cg(&g, prm->eps, p.Y, p.X, ld, k, prm->tol, prm->max_iter,
+                                   iters + c0, relres + c0, p.cg_ws, p.cg_bytes,
+                                   reinterpret_cast<erc_stream>(s));
+    if (st == ERC_ERR_NOT_CONVERGED) {
+      worst = st;
+    } else if (st != ERC_OK) {
+      return st;
+    }
+    ERC_TRY(erc_edge_resistance(&g, p.X, ld, k, R, reinterpret_cast<erc_stream>(s)));
+  }
+  ERC_TRY(erc_curvature(&g, R, p_node, kappa, reinterpret_cast<erc_stream>(s)));
+  ERC_TRY(erc_sampling_probs(&g, kappa, prm->eta, prob_node, prob_edge, p.aux_ws, p.aux_bytes,
+                             reinterpret_cast<erc_stream>(s)));
+  if (worst != ERC_OK) return set_error(worst, "some CG columns reached max_iter");
+  return ERC_OK;
+}
+
+erc_status check_params(const erc_params* prm, int32_t n, int64_t m_in) {
+  ERC_REQUIRE(prm, "params is null");
+  ERC_REQUIRE(prm->K >= 1, "K must be >= 1");
+  ERC_REQUIRE(prm->kc >= 1 && prm->kc <= MAX_LD, "kc must be in [1, %d]", MAX_LD);
+  ERC_REQUIRE(prm->kc % 4 == 0 || prm->kc >= prm->K, "kc must be a multiple of 4 when K > kc");
+  ERC_REQUIRE(n >= 1 && m_in >= 0, "bad n / m_in");
+  return ERC_OK;
+}
+
+}  // namespace
+}  // namespace erc
+
+using namespace erc;
+
+extern "C" const char* erc_version(void) { return "erc-gb300 0.1 (sm_103a)"; }
+extern "C" const char* erc_last_error(void) { return g_err; }
+
+extern "C" size_t erc_run_workspace_size(int32_t n, int64_t m_in, int32_t kc) {
+  if (n < 1 || m_in < 0 || kc < 1) return 0;
+  Arena a(nullptr);
+  RunPlan p;
+  plan_run(a, p, n, m_in, kc);
+  return a.used + 256;
+}
+
+extern "C" erc_status erc_run(const erc_params* prm, int32_t n, const int32_t* src,
+                              const int32_t* dst, const float* w, int64_t m_in, int64_t* m_out,
+                              int32_t* eu, int32_t* ev, float* R, float* p_node, float* kappa,
+                              float* prob_node, float* prob_edge, int32_t* iters, float* relres,
+                              void* ws, size_t ws_bytes, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_params(prm, n, m_in));
+  ERC_REQUIRE(m_out && eu && ev && R && p_node && kappa && prob_node && prob_edge && iters &&
+                  relres,
+              "output pointers are required");
+  if (ws_bytes < erc_run_workspace_size(n, m_in, prm->kc))
+    return set_error(ERC_ERR_CAPACITY, "workspace too small");
+  Arena a(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  RunPlan p;
+  plan_run(a, p, n, m_in, prm->kc);
+  return run_device(prm, n, src, dst, w, m_in, m_out, eu, ev, R, p_node, kappa, prob_node,
+                    prob_edge, iters, relres, p, as_stream(stream));
+}
+
+namespace {
+struct HostIo {
+  int32_t *src, *dst;
+  float* w;
+  int32_t *eu, *ev;
+  float *R, *p, *kappa, *pn, *pe, *relres;
+  int32_t* iters;
+};
+void plan_host_io(Arena& a, HostIo& h, int32_t n, int64_t m_in, int32_t K) {
+  h.src = a.take<int32_t>(m_in);
+  h.dst = a.take<int32_t>(m_in);
+  h.w = a.take<float>(m_in);
+  h.eu = a.take<int32_t>(m_in);
+  h.ev = a.take<int32_t>(m_in);
+  h.R = a.take<float>(m_in);
+  h.kappa = a.take<float>(m_in);
+  h.pe = a.take<float>(m_in);
+  h.p = a.take<float>(n);
+  h.pn = a.take<float>(n);
+  h.iters = a.take<int32_t>(K);
+  h.relres = a.take<float>(K);
+}
+}  // namespace
+
+extern "C" size_t erc_run_host_workspace_size(int32_t n, int64_t m_in, int32_t kc, int32_t K) {
+  if (n < 1 || m_in < 0 || kc < 1 || K < 1) return 0;
+  Arena a(nullptr);
+  HostIo h;
+  plan_host_io(a, h, n, m_in, K);
+  RunPlan p;
+  plan_run(a, p, n, m_in, kc);
+  return a.used + 256;
+}
+
+extern "C" erc_status erc_run_host(const erc_params* prm, int32_t n, const int32_t* src,
+                                   const int32_t* dst, const float* w, int64_t m_in,
+                                   int64_t* m_out, int32_t* eu, int32_t* ev, float* R,
+                                   float* p_node, float* kappa, float* prob_node,
+                                   float* prob_edge, int32_t* iters, float* relres, void* ws,
+                                   size_t ws_bytes, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_params(prm, n, m_in));
+  ERC_REQUIRE(m_in == 0 || (src && dst), "src and dst are required");
+  ERC_REQUIRE(m_out && eu && ev && R && p_node && kappa && prob_node && prob_edge && iters &&
+                  relres,
+              "output pointers are required");
+  if (ws_bytes < erc_run_host_workspace_size(n, m_in, prm->kc, prm->K))
+    return set_error(ERC_ERR_CAPACITY, "workspace too small");
+  cudaStream_t s = as_stream(stream);
+  Arena a(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  HostIo d;
+  plan_host_io(a, d, n, m_in, prm->K);
+  RunPlan p;
+  plan_run(a, p, n, m_in, prm->kc);
+  const size_t mi4 = (size_t)m_in * 4;
+  if (m_in > 0) {
+    ERC_CUDA(cudaMemcpyAsync(d.src, src, mi4, cudaMemcpyHostToDevice, s));
+    ERC_CUDA(cudaMemcpyAsync(d.dst, dst, mi4, cudaMemcpyHostToDevice, s));
+    if (w) ERC_CUDA(cudaMemcpyAsync(d.w, w, mi4, cudaMemcpyHostToDevice, s));
+  }
+  erc_status st = run_device(prm, n, d.src, d.dst, w ? d.w : nullptr, m_in, m_out, d.eu, d.ev,
+                             d.R, d.p, d.kappa, d.pn, d.pe, d.iters, d.relres, p, s);
+  if (st != ERC_OK && st != ERC_ERR_NOT_CONVERGED) return st;
+  const size_t m4 = (size_t)(*m_out) * 4, n4 = (size_t)n * 4, k4 = (size_t)prm->K * 4;
+  if (m4) {
+    ERC_CUDA(cudaMemcpyAsync(eu, d.eu, m4, cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaMemcpyAsync(ev, d.ev, m4, cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaMemcpyAsync(R, d.R, m4, cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaMemcpyAsync(kappa, d.kappa, m4, cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaMemcpyAsync(prob_edge, d.pe, m4, cudaMemcpyDeviceToHost, s));
+  }
+  ERC_CUDA(cudaMemcpyAsync(p_node, d.p, n4, cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(prob_node, d.pn, n4, cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(iters, d.iters, k4, cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(relres, d.relres, k4, cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaStreamSynchronize(s));
+  return st;
+}

@@ -1,0 +1,687 @@
+// cg.cu -- column-wise CG on L_eps X = Y (Eq. 5, §3.1.3, Algorithm 1) and the operator
+// L_eps P = eps P + (D - A) P it iterates on.
+//
+// One CG iteration is three kernels over the row-major n x ld block:
+//   k_spmm<MODE_STEP>  AP = L_eps P (warp-per-row gather of neighbour rows, float4 along the
+//                      columns), per-column p.Ap partials; the last block forms alpha = rr / pAp.
+//   k_update_xr        x += alpha p, r -= alpha Ap, per-column r.r; the last block forms beta,
+//                      counts the iteration and retires converged columns.
+//   k_update_p         p = r + beta p for the columns still active.
+// Reductions are deterministic (fixed order, float-pair accumulation).  A run of S iterations
+// is captured once into a CUDA graph and relaunched; kernels return at once when no column is
+// active, so the host only polls the "any active" flag between graph launches.
+#include <cstring>
+#include <mutex>
+
+#include "erc_internal.cuh"
+
+namespace erc {
+namespace {
+
+constexpr int T = 256;
+constexpr int WARPS = T / 32;
+enum { MODE_STEP = 0, MODE_APPLY = 1, MODE_RESID = 2 };
+
+struct CgWork {
+  float *R, *P, *AP;
+  float *alpha, *beta;
+  double *rr, *yy;
+  int *active, *conv, *iters;
+  int* flags;  // [0] any column active  [1] numeric trouble  [2] unconverged columns
+  ColReduce cr;
+};
+
+void plan_cg(Arena& a, CgWork& w, int32_t n, int32_t ld) {
+  const size_t blk = (size_t)n * ld;
+  w.R = a.take<float>(blk);
+  w.P = a.take<float>(blk);
+  w.AP = a.take<float>(blk);
+  w.alpha = a.take<float>(ld);
+  w.beta = a.take<float>(ld);
+  w.rr = a.take<double>(ld);
+  w.yy = a.take<double>(ld);
+  w.active = a.take<int>(ld);
+  w.conv = a.take<int>(ld);
+  w.iters = a.take<int>(ld);
+  w.flags = a.take<int>(8);
+  plan_colreduce(a, w.cr, ld);
+}
+
+struct SpmmArgs {
+  const int64_t* row_ptr;
+  const int32_t* col;
+  const float* val;
+  int32_t n, ld, kc;
+  float eps;
+  const float* P;  // operand: P (step/apply) or X (residual)
+  float* AP;       // output of step/apply
+  const float* Y;  // residual mode
+  ColReduce cr;
+  float* alpha;
+  const double* rr;
+  int* active;
+  int* flags;
+  double* pap_out;  // apply mode, may be null
+  const double* yy;
+  const int* iters;
+  const int* conv;
+  float* relres_out;
+  int32_t* iters_out;
+};
+
+// per-warp then per-block combination of per-thread column partials of a row-group kernel
+template <int LPR, int VPL>
+__device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], float2* sbuf,
+                                                        float2* scratch, int ld) {
+#pragma unroll
+  for (int off = LPR; off < 32; off <<= 1) {
+#pragma unroll
+    for (int v = 0; v < VPL; ++v)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        float2 o;
+        o.x = __shfl_xor_sync(0xffffffffu, d[v][t].x, off);
+        o.y = __shfl_xor_sync(0xffffffffu, d[v][t].y, off);
+        d[v][t] = df_add(d[v][t], o);
+      }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int cb = 0; cb < ld; cb += 256) {
+    if (lane < LPR) {
+#pragma unroll
+      for (int v = 0; v < VPL; ++v)
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int c = 4 * (lane + LPR * v) + t;
+          if (c >= cb && c < cb + 256 && c < ld) scratch[warp * 256 + (c - cb)] = d[v][t];
+        }
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < 256 && cb + c < ld; c += blockDim.x) {
+      float2 acc = make_float2(0.f, 0.f);
+      for (int w = 0; w < WARPS; ++w) acc = df_add(acc, scratch[w * 256 + c]);
+      sbuf[cb + c] = acc;
+    }
+    __syncthreads();
+  }
+}
+
+__device__ __forceinline__ float4 ld_f4(const float* p) {
+  return __ldg(reinterpret_cast<const float4*>(p));
+}
+
+template <int LPR, int VPL, bool WEIGHTED, int MODE>
+__global__ void __launch_bounds__(T) k_spmm(SpmmArgs a) {
+  if (MODE == MODE_STEP && *(volatile int*)a.flags == 0) return;
+  __shared__ float2 sbuf[MAX_LD];
+  __shared__ float2 scratch[WARPS * 256];
+  constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
+  const int gl = threadIdx.x & (LPR - 1);
+  const int gpb = T / LPR;
+  const int nvec = a.ld >> 2;
+  const unsigned gm = group_mask<LPR>();
+  float2 dot[VPL][4];
+#pragma unroll
+  for (int v = 0; v < VPL; ++v)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
+
+  for (int64_t u = (int64_t)blockIdx.x * gpb + threadIdx.x / LPR; u < a.n;
+       u += (int64_t)gridDim.x * gpb) {
+    float4 pu[VPL], acc[VPL];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      pu[v] = q < nvec ? ld_f4(a.P + (size_t)u * a.ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+    for (int64_t jb = j0; jb < j1; jb += LPR) {
+      const int64_t jj = jb + gl;
+      int32_t cidx = 0;
+      float wv = 1.f;
+      if (jj < j1) {
+        cidx = __ldg(a.col + jj);
+        if (WEIGHTED) wv = __ldg(a.val + jj);
+      }
+      const int cnt = (int)min((int64_t)LPR, j1 - jb);
+      int t = 0;
+      for (; t + U <= cnt; t += U) {
+        int cj[U];
+        float wj[U];
+        float4 pv[U][VPL];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          cj[k] = __shfl_sync(gm, cidx, t + k, LPR);
+          wj[k] = WEIGHTED ? __shfl_sync(gm, wv, t + k, LPR) : 1.f;
+        }
+#pragma unroll
+        for (int k = 0; k < U; ++k)
+#pragma unroll
+          for (int v = 0; v < VPL; ++v) {
+            const int q = gl + LPR * v;
+            pv[k][v] = q < nvec ? ld_f4(a.P + (size_t)cj[k] * a.ld + 4 * q)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+#pragma unroll
+        for (int k = 0; k < U; ++k)
+#pragma unroll
+          for (int v = 0; v < VPL; ++v) {
+            acc[v].x = fmaf(wj[k], pu[v].x - pv[k][v].x, acc[v].x);
+            acc[v].y = fmaf(wj[k], pu[v].y - pv[k][v].y, acc[v].y);
+            acc[v].z = fmaf(wj[k], pu[v].z - pv[k][v].z, acc[v].z);
+            acc[v].w = fmaf(wj[k], pu[v].w - pv[k][v].w, acc[v].w);
+          }
+      }
+      for (; t < cnt; ++t) {
+        const int c1 = __shfl_sync(gm, cidx, t, LPR);
+        const float w1 = WEIGHTED ? __shfl_sync(gm, wv, t, LPR) : 1.f;
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int q = gl + LPR * v;
+          if (q < nvec) {
+            const float4 p1 = ld_f4(a.P + (size_t)c1 * a.ld + 4 * q);
+            acc[v].x = fmaf(w1, pu[v].x - p1.x, acc[v].x);
+            acc[v].y = fmaf(w1, pu[v].y - p1.y, acc[v].y);
+            acc[v].z = fmaf(w1, pu[v].z - p1.z, acc[v].z);
+            acc[v].w = fmaf(w1, pu[v].w - p1.w, acc[v].w);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q >= nvec) continue;
+      float4 o;  // L_eps p = eps p_u + sum_v w_uv (p_u - p_v)
+      o.x = fmaf(a.eps, pu[v].x, acc[v].x);
+      o.y = fmaf(a.eps, pu[v].y, acc[v].y);
+      o.z = fmaf(a.eps, pu[v].z, acc[v].z);
+      o.w = fmaf(a.eps, pu[v].w, acc[v].w);
+      if (MODE == MODE_RESID) {
+        const float4 y = ld_f4(a.Y + (size_t)u * a.ld + 4 * q);
+        const int cb = 4 * q;
+        o.x = cb + 0 < a.kc ? y.x - o.x : 0.f;
+        o.y = cb + 1 < a.kc ? y.y - o.y : 0.f;
+        o.z = cb + 2 < a.kc ? y.z - o.z : 0.f;
+        o.w = cb + 3 < a.kc ? y.w - o.w : 0.f;
+        dot[v][0] = df_fma(dot[v][0], o.x, o.x);
+        dot[v][1] = df_fma(dot[v][1], o.y, o.y);
+        dot[v][2] = df_fma(dot[v][2], o.z, o.z);
+        dot[v][3] = df_fma(dot[v][3], o.w, o.w);
+      } else {
+        reinterpret_cast<float4*>(a.AP + (size_t)u * a.ld)[q] = o;
+        dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
+        dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
+        dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
+        dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
+      }
+    }
+  }
+  if (MODE == MODE_APPLY && a.pap_out == nullptr) return;
+
+  block_partials_rowgroup<LPR, VPL>(dot, sbuf, scratch, a.ld);
+  if (!grid_colreduce(a.cr, sbuf, sbuf, a.ld)) return;
+  for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
+    const double v = df_value(sbuf[c]);
+    if (MODE == MODE_STEP) {
+      float al = 0.f;
+      if (a.active[c]) {
+        const double q = a.rr[c] / v;
+        if (!(v > 0.0) || !isfinite(q)) {
+          a.active[c] = 0;
+          atomicOr(&a.flags[1], 1);
+        } else {
+          al = (float)q;
+        }
+      }
+      a.alpha[c] = al;
+    } else if (MODE == MODE_APPLY) {
+      if (c < a.kc) a.pap_out[c] = v;
+    } else {
+      if (c < a.kc) {
+        const double y2 = a.yy[c];
+        a.relres_out[c] = y2 > 0.0 ? (float)sqrt(v / y2) : 0.f;
+        a.iters_out[c] = a.iters[c];
+        if (!a.conv[c]) atomicAdd(&a.flags[2], 1);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- vector kernels
+// Each thread keeps one column quad q (4 columns) and walks the rows, so its partial sums
+// belong to fixed columns.  Threads per block = nvec * (256 / nvec).
+struct VecArgs {
+  int32_t n, ld, kc;
+  double tol2;
+  int32_t max_iter;
+  const float* Y;
+  float *X, *R, *P, *AP;
+  float *alpha, *beta;
+  double *rr, *yy;
+  int *active, *conv, *iters, *flags;
+  ColReduce cr;
+};
+
+__device__ __forceinline__ void block_partials_quad(const float2 (&d)[4], float2* red,
+                                                    float2* sbuf, int ld, int nvec) {
+#pragma unroll
+  for (int t = 0; t < 4; ++t) red[threadIdx.x * 4 + t] = d[t];
+  __syncthreads();
+  const int rb = blockDim.x / nvec;
+  for (int c = threadIdx.x; c < ld; c += blockDim.x) {
+    const int q = c >> 2, t = c & 3;
+    float2 acc = make_float2(0.f, 0.f);
+    for (int r = 0; r < rb; ++r) acc = df_add(acc, red[(r * nvec + q) * 4 + t]);
+    sbuf[c] = acc;
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
+  __shared__ float2 red[T * 4];
+  __shared__ float2 sbuf[MAX_LD];
+  const int nvec = a.ld >> 2, rb = blockDim.x / nvec;
+  const int q = threadIdx.x % nvec;
+  float2 d[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
+  const int cb = 4 * q;
+  for (int64_t row = (int64_t)blockIdx.x * rb + threadIdx.x / nvec; row < a.n;
+       row += (int64_t)gridDim.x * rb) {
+    const size_t i = (size_t)row * a.ld + cb;
+    float4 y = ld_f4(a.Y + i);
+    if (cb + 0 >= a.kc) y.x = 0.f;
+    if (cb + 1 >= a.kc) y.y = 0.f;
+    if (cb + 2 >= a.kc) y.z = 0.f;
+    if (cb + 3 >= a.kc) y.w = 0.f;
+    *reinterpret_cast<float4*>(a.R + i) = y;
+    *reinterpret_cast<float4*>(a.P + i) = y;
+    *reinterpret_cast<float4*>(a.X + i) = make_float4(0.f, 0.f, 0.f, 0.f);
+    d[0] = df_fma(d[0], y.x, y.x);
+    d[1] = df_fma(d[1], y.y, y.y);
+    d[2] = df_fma(d[2], y.z, y.z);
+    d[3] = df_fma(d[3], y.w, y.w);
+  }
+  block_partials_quad(d, red, sbuf, a.ld, nvec);
+  if (!grid_colreduce(a.cr, sbuf, sbuf, a.ld)) return;
+  int any = 0;
+  for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
+    const double v = df_value(sbuf[c]);
+    a.yy[c] = v;
+    a.rr[c] = v;
+    a.iters[c] = 0;
+    a.alpha[c] = 0.f;
+    a.beta[c] = 0.f;
+    int act = 0, cv = 1;
+    if (c < a.kc) {
+      if (!isfinite(v)) {
+        atomicOr(&a.flags[1], 1);
+        cv = 0;
+      } else if (v > 0.0 && !(v <= a.tol2 * v)) {
+        act = 1;
+        cv = 0;
+      }
+    }
+    a.active[c] = act;
+    a.conv[c] = cv;
+    any |= act;
+  }
+  any = __syncthreads_or(any);
+  if (threadIdx.x == 0) a.flags[0] = any;
+}
+
+__global__ void __launch_bounds__(T) k_update_xr(VecArgs a) {
+  if (*(volatile int*)a.flags == 0) return;
+  __shared__ float2 red[T * 4];
+  __shared__ float2 sbuf[MAX_LD];
+  const int nvec = a.ld >> 2, rb = blockDim.x / nvec;
+  const int q = threadIdx.x % nvec;
+  const float4 al = *reinterpret_cast<const float4*>(a.alpha + 4 * q);
+  float2 d[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
+  if (al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f) {
+    for (int64_t row = (int64_t)blockIdx.x * rb + threadIdx.x / nvec; row < a.n;
+         row += (int64_t)gridDim.x * rb) {
+      const size_t i = (size_t)row * a.ld + 4 * q;
+      float4 x = *reinterpret_cast<const float4*>(a.X + i);
+      float4 r = *reinterpret_cast<const float4*>(a.R + i);
+      const float4 p = *reinterpret_cast<const float4*>(a.P + i);
+      const float4 ap = *reinterpret_cast<const float4*>(a.AP + i);
+      x.x = fmaf(al.x, p.x, x.x);
+      x.y = fmaf(al.y, p.y, x.y);
+      x.z = fmaf(al.z, p.z, x.z);
+      x.w = fmaf(al.w, p.w, x.w);
+      r.x = fmaf(-al.x, ap.x, r.x);
+      r.y = fmaf(-al.y, ap.y, r.y);
+      r.z = fmaf(-al.z, ap.z, r.z);
+      r.w = fmaf(-al.w, ap.w, r.w);
+      *reinterpret_cast<float4*>(a.X + i) = x;
+      *reinterpret_cast<float4*>(a.R + i) = r;
+      d[0] = df_fma(d[0], r.x, r.x);
+      d[1] = df_fma(d[1], r.y, r.y);
+      d[2] = df_fma(d[2], r.z, r.z);
+      d[3] = df_fma(d[3], r.w, r.w);
+    }
+  }
+  block_partials_quad(d, red, sbuf, a.ld, nvec);
+  if (!grid_colreduce(a.cr, sbuf, sbuf, a.ld)) return;
+  int any = 0;
+  for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
+    float be = 0.f;
+    if (a.active[c]) {
+      const double rn = df_value(sbuf[c]);
+      const int it = a.iters[c] + 1;
+      a.iters[c] = it;
+      if (!isfinite(rn)) {
+        a.active[c] = 0;
+        atomicOr(&a.flags[1], 1);
+      } else {
+        be = (float)(rn / a.rr[c]);
+        a.rr[c] = rn;
+        if (rn <= a.tol2 * a.yy[c]) {
+          a.conv[c] = 1;
+          a.active[c] = 0;
+        } else if (it >= a.max_iter) {
+          a.active[c] = 0;
+        }
+      }
+    }
+    a.beta[c] = be;
+    any |= a.active[c];
+  }
+  any = __syncthreads_or(any);
+  if (threadIdx.x == 0) a.flags[0] = any;
+}
+
+__global__ void __launch_bounds__(T) k_update_p(VecArgs a) {
+  if (*(volatile int*)a.flags == 0) return;
+  const int nvec = a.ld >> 2, rb = blockDim.x / nvec;
+  const int q = threadIdx.x % nvec;
+  const int4 act = *reinterpret_cast<const int4*>(a.active + 4 * q);
+  if (!(act.x | act.y | act.z | act.w)) return;
+  const float4 be = *reinterpret_cast<const float4*>(a.beta + 4 * q);
+  for (int64_t row = (int64_t)blockIdx.x * rb + threadIdx.x / nvec; row < a.n;
+       row += (int64_t)gridDim.x * rb) {
+    const size_t i = (size_t)row * a.ld + 4 * q;
+    const float4 r = *reinterpret_cast<const float4*>(a.R + i);
+    float4 p = *reinterpret_cast<const float4*>(a.P + i);
+    if (act.x) p.x = fmaf(be.x, p.x, r.x);
+    if (act.y) p.y = fmaf(be.y, p.y, r.y);
+    if (act.z) p.z = fmaf(be.z, p.z, r.z);
+    if (act.w) p.w = fmaf(be.w, p.w, r.w);
+    *reinterpret_cast<float4*>(a.P + i) = p;
+  }
+}
+
+// ---------------------------------------------------------------------------- launch helpers
+inline int vec_threads(int nvec) { return nvec * (T / nvec); }
+
+template <int MODE>
+erc_status launch_spmm(const SpmmArgs& a, cudaStream_t s) {
+  return dispatch_shape(a.ld / 4, [&](auto lpr, auto vpl) -> erc_status {
+    constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
+    const int grid = grid_for(a.n, T / LPR);
+    if (a.val)
+      k_spmm<LPR, VPL, true, MODE><<<grid, T, 0, s>>>(a);
+    else
+      k_spmm<LPR, VPL, false, MODE><<<grid, T, 0, s>>>(a);
+    ERC_CUDA(cudaGetLastError());
+    return ERC_OK;
+  });
+}
+
+inline int vec_grid(int32_t n, int nvec) { return grid_for(n, vec_threads(nvec) / nvec); }
+
+erc_status launch_iteration(const SpmmArgs& sa, const VecArgs& va, cudaStream_t s) {
+  ERC_TRY(launch_spmm<MODE_STEP>(sa, s));
+  const int nvec = va.ld / 4;
+  k_update_xr<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
+  ERC_CUDA(cudaGetLastError());
+  k_update_p<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
+  ERC_CUDA(cudaGetLastError());
+  return ERC_OK;
+}
+
+// ---------------------------------------------------------------------------- graph cache
+struct GraphKey {
+  const void* ptr[12];
+  long long num[8];
+  bool operator==(const GraphKey& o) const {
+    for (int i = 0; i < 12; ++i)
+      if (ptr[i] != o.ptr[i]) return false;
+    for (int i = 0; i < 8; ++i)
+      if (num[i] != o.num[i]) return false;
+    return true;
+  }
+};
+struct GraphEntry {
+  GraphKey key;
+  cudaGraphExec_t exec = nullptr;
+  unsigned long long stamp = 0;
+};
+constexpr int CACHE = 16;
+std::mutex g_mu;
+GraphEntry g_cache[CACHE];
+unsigned long long g_clock = 0;
+
+cudaStream_t capture_stream() {
+  static thread_local cudaStream_t cs[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return nullptr;
+  if (!cs[dev]) cudaStreamCreateWithFlags(&cs[dev], cudaStreamNonBlocking);
+  return cs[dev];
+}
+
+erc_status iteration_graph(const SpmmArgs& sa, const VecArgs& va, int S, cudaGraphExec_t* out) {
+  int dev = 0;
+  ERC_CUDA(cudaGetDevice(&dev));
+  GraphKey k{};
+  const void* ptrs[12] = {sa.row_ptr, sa.col, sa.val, sa.P, sa.AP, va.X, va.R, va.alpha,
+                          va.active, va.flags, sa.cr.part1, va.Y};
+  for (int i = 0; i < 12; ++i) k.ptr[i] = ptrs[i];
+  int eps_bits = 0;
+  long long tol_bits = 0;
+  memcpy(&eps_bits, &sa.eps, sizeof eps_bits);
+  memcpy(&tol_bits, &va.tol2, sizeof tol_bits);
+  long long nums[8] = {sa.n, sa.ld, sa.kc, eps_bits, tol_bits, va.max_iter, S, dev};
+  for (int i = 0; i < 8; ++i) k.num[i] = nums[i];
+  std::lock_guard<std::mutex> lock(g_mu);
+  ++g_clock;
+  int victim = 0;
+  for (int i = 0; i < CACHE; ++i) {
+    if (g_cache[i].exec && g_cache[i].key == k) {
+      g_cache[i].stamp = g_clock;
+      *out = g_cache[i].exec;
+      return ERC_OK;
+    }
+    if (g_cache[i].stamp < g_cache[victim].stamp) victim = i;
+  }
+  cudaStream_t cs = capture_stream();
+  if (!cs) return set_error(ERC_ERR_CUDA, "no capture stream");
+  ERC_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  erc_status st = ERC_OK;
+  for (int i = 0; i < S && st == ERC_OK; ++i) st = launch_iteration(sa, va, cs);
+  cudaGraph_t graph = nullptr;
+  cudaError_t ce = cudaStreamEndCapture(cs, &graph);
+  if (st != ERC_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return st;
+  }
+  if (ce != cudaSuccess) return set_error(ERC_ERR_CUDA, "graph capture: %s", cudaGetErrorString(ce));
+  cudaGraphExec_t exec = nullptr;
+  ce = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (ce != cudaSuccess)
+    return set_error(ERC_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(ce));
+  if (g_cache[victim].exec) cudaGraphExecDestroy(g_cache[victim].exec);
+  g_cache[victim].key = k;
+  g_cache[victim].exec = exec;
+  g_cache[victim].stamp = g_clock;
+  *out = exec;
+  return ERC_OK;
+}
+
+int iterations_per_poll(const erc_graph* g, int ld) {
+  const double bytes = (double)(2 * g->m + g->n) * ld * 4.0;  // gathered + streamed per iteration
+  if (bytes < 64e6) return 32;
+  if (bytes < 1e9) return 8;
+  return 2;
+}
+
+erc_status check_block(const erc_graph* g, const float* p, int ld, const char* name) {
+  ERC_REQUIRE(p && (reinterpret_cast<uintptr_t>(p) & 15) == 0, "%s must be 16-byte aligned", name);
+  (void)g;
+  (void)ld;
+  return ERC_OK;
+}
+
+}  // namespace
+}  // namespace erc
+
+using namespace erc;
+
+extern "C" size_t erc_batched_cg_workspace_size(int32_t n, int32_t ld) {
+  if (n < 1 || ld < 4) return 0;
+  Arena a(nullptr);
+  CgWork w;
+  plan_cg(a, w, n, ld);
+  return a.used + 256;
+}
+
+extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* X,
+                                     int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                     int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                     erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
+  ERC_REQUIRE(eps > 0.f && isfinite(eps), "eps must be positive");
+  ERC_REQUIRE(tol >= 0.f && isfinite(tol), "tol must be finite and >= 0");
+  ERC_REQUIRE(max_iter >= 1, "max_iter must be >= 1");
+  ERC_REQUIRE(iters && relres, "iters and relres are required");
+  ERC_TRY(check_block(g, Y, ld, "Y"));
+  ERC_TRY(check_block(g, X, ld, "X"));
+  if (ws_bytes < erc_batched_cg_workspace_size(g->n, ld))
+    return set_error(ERC_ERR_CAPACITY, "workspace too small");
+  cudaStream_t s = as_stream(stream);
+  Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  CgWork w;
+  plan_cg(ar, w, g->n, ld);
+  ERC_CUDA(cudaMemsetAsync(w.cr.cnt, 0, colreduce_counter_bytes(), s));
+  ERC_CUDA(cudaMemsetAsync(w.flags, 0, 8 * sizeof(int), s));
+
+  VecArgs va{};
+  va.n = g->n;
+  va.ld = ld;
+  va.kc = kc;
+  va.tol2 = (double)tol * (double)tol;
+  va.max_iter = max_iter;
+  va.Y = Y;
+  va.X = X;
+  va.R = w.R;
+  va.P = w.P;
+  va.AP = w.AP;
+  va.alpha = w.alpha;
+  va.beta = w.beta;
+  va.rr = w.rr;
+  va.yy = w.yy;
+  va.active = w.active;
+  va.conv = w.conv;
+  va.iters = w.iters;
+  va.flags = w.flags;
+  va.cr = w.cr;
+
+  SpmmArgs sa{};
+  sa.row_ptr = g->row_ptr;
+  sa.col = g->col;
+  sa.val = g->val;
+  sa.n = g->n;
+  sa.ld = ld;
+  sa.kc = kc;
+  sa.eps = eps;
+  sa.P = w.P;
+  sa.AP = w.AP;
+  sa.Y = Y;
+  sa.cr = w.cr;
+  sa.alpha = w.alpha;
+  sa.rr = w.rr;
+  sa.active = w.active;
+  sa.flags = w.flags;
+  sa.yy = w.yy;
+  sa.iters = w.iters;
+  sa.conv = w.conv;
+  sa.relres_out = relres;
+  sa.iters_out = iters;
+
+  const int nvec = ld / 4;
+  k_cg_init<<<vec_grid(g->n, nvec), vec_threads(nvec), 0, s>>>(va);
+  ERC_CUDA(cudaGetLastError());
+
+  const int S = iterations_per_poll(g, ld);
+  cudaGraphExec_t exec = nullptr;
+  ERC_TRY(iteration_graph(sa, va, S, &exec));
+  int done = 0;
+  int h_any = 1;
+  while (done < max_iter) {
+    ERC_CUDA(cudaGraphLaunch(exec, s));
+    done += S;
+    ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
+    ERC_CUDA(cudaStreamSynchronize(s));
+    if (!h_any) break;
+  }
+
+  // true residual of the returned iterate, plus the per-column outputs
+  SpmmArgs ra = sa;
+  ra.P = X;
+  ERC_TRY(launch_spmm<MODE_RESID>(ra, s));
+  int h_flags[3] = {0, 0, 0};
+  ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 3 * sizeof(int), cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaStreamSynchronize(s));
+  if (h_flags[1]) return set_error(ERC_ERR_NUMERIC, "non-finite or non-positive CG scalar");
+  if (h_flags[2])
+    return set_error(ERC_ERR_NOT_CONVERGED, "%d of %d columns reached max_iter=%d", h_flags[2],
+                     kc, max_iter);
+  return ERC_OK;
+}
+
+extern "C" size_t erc_laplacian_apply_workspace_size(int32_t n, int32_t ld) {
+  (void)n;
+  if (ld < 4) return 0;
+  Arena a(nullptr);
+  ColReduce cr;
+  plan_colreduce(a, cr, ld);
+  return a.used + 256;
+}
+
+extern "C" erc_status erc_laplacian_apply(const erc_graph* g, float eps, const float* P,
+                                          float* AP, int32_t ld, int32_t kc, double* pAp,
+                                          void* ws, size_t ws_bytes, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
+  ERC_REQUIRE(eps >= 0.f && isfinite(eps), "eps must be finite and >= 0");
+  ERC_TRY(check_block(g, P, ld, "P"));
+  ERC_TRY(check_block(g, AP, ld, "AP"));
+  cudaStream_t s = as_stream(stream);
+  SpmmArgs sa{};
+  sa.row_ptr = g->row_ptr;
+  sa.col = g->col;
+  sa.val = g->val;
+  sa.n = g->n;
+  sa.ld = ld;
+  sa.kc = kc;
+  sa.eps = eps;
+  sa.P = P;
+  sa.AP = AP;
+  sa.pap_out = pAp;
+  if (pAp) {
+    if (ws_bytes < erc_laplacian_apply_workspace_size(g->n, ld))
+      return set_error(ERC_ERR_CAPACITY, "workspace too small");
+    Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+    plan_colreduce(ar, sa.cr, ld);
+    ERC_CUDA(cudaMemsetAsync(sa.cr.cnt, 0, colreduce_counter_bytes(), s));
+  }
+  return launch_spmm<MODE_APPLY>(sa, s);
+}

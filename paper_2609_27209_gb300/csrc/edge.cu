@@ -1,0 +1,359 @@
+// edge.cu -- the O(n + m) tail of the path:
+//   erc_edge_resistance  R_e += sum_c (X_u,c - X_v,c)^2 over a column batch   (Eq. 6, Algorithm 1)
+//   erc_curvature        p_u = 1 - 1/2 sum_v w_uv R_uv, kappa_uv = 2 (p_u + p_v) / R_uv (Eq. 2)
+//   erc_sampling_probs   Eq. 7 (with the uniform fallback), Eq. 8, normalisation (§3.2)
+#include <cfloat>
+
+#include "erc_internal.cuh"
+
+namespace erc {
+namespace {
+
+constexpr int T = 256;
+
+__device__ __forceinline__ float4 ld_f4(const float* p) {
+  return __ldg(reinterpret_cast<const float4*>(p));
+}
+
+// One group of LPR lanes walks a segment of consecutive canonical edges.  Edges are sorted by
+// their smaller endpoint, so X_u is reloaded only when u changes; the group owns each R_e it
+// touches, so the accumulation needs no atomics.
+template <int LPR, int VPL>
+__global__ void __launch_bounds__(T)
+    k_edge_resistance(const int32_t* __restrict__ eu, const int32_t* __restrict__ ev, int64_t m,
+                      const float* __restrict__ X, int32_t ld, int32_t kc, float* __restrict__ R) {
+  constexpr int SEG = 32;
+  const int gl = threadIdx.x & (LPR - 1);
+  const int gpb = T / LPR;
+  const int nvec = ld >> 2;
+  const unsigned gm = group_mask<LPR>();
+  const int64_t nseg = (m + SEG - 1) / SEG;
+  for (int64_t sg = (int64_t)blockIdx.x * gpb + threadIdx.x / LPR; sg < nseg;
+       sg += (int64_t)gridDim.x * gpb) {
+    const int64_t e0 = sg * SEG, e1 = min(m, e0 + SEG);
+    int32_t cu = -1;
+    float4 xu[VPL];
+    for (int64_t e = e0; e < e1; ++e) {
+      const int32_t u = __ldg(eu + e), v = __ldg(ev + e);
+      if (u != cu) {
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) {
+          const int q = gl + LPR * k;
+          xu[k] = q < nvec ? ld_f4(X + (size_t)u * ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        cu = u;
+      }
+      float s = 0.f;
+#pragma unroll
+      for (int k = 0; k < VPL; ++k) {
+        const int q = gl + LPR * k;
+        if (q < nvec) {
+          const float4 xv = ld_f4(X + (size_t)v * ld + 4 * q);
+          const int cb = 4 * q;
+          const float dx = cb + 0 < kc ? xu[k].x - xv.x : 0.f;
+          const float dy = cb + 1 < kc ? xu[k].y - xv.y : 0.f;
+          const float dz = cb + 2 < kc ? xu[k].z - xv.z : 0.f;
+          const float dw = cb + 3 < kc ? xu[k].w - xv.w : 0.f;
+          s = fmaf(dx, dx, s);
+          s = fmaf(dy, dy, s);
+          s = fmaf(dz, dz, s);
+          s = fmaf(dw, dw, s);
+        }
+      }
+#pragma unroll
+      for (int off = LPR / 2; off > 0; off >>= 1) s += __shfl_xor_sync(gm, s, off, LPR);
+      if (gl == 0) R[e] += s;
+    }
+  }
+}
+
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+// p_u = 1 - 1/2 sum_{slots j of row u} w_j R[eid_j]; a warp per row, float64 sums
+template <bool WEIGHTED>
+__global__ void __launch_bounds__(T)
+    k_node_curvature(const int64_t* __restrict__ row_ptr, const float* __restrict__ val,
+                     const int32_t* __restrict__ eid, const float* __restrict__ R, int32_t n,
+                     float* __restrict__ p) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wpb = T / 32;
+  for (int64_t u = (int64_t)blockIdx.x * wpb + threadIdx.x / 32; u < n;
+       u += (int64_t)gridDim.x * wpb) {
+    double acc = 0.0;
+    for (int64_t j = row_ptr[u] + lane; j < row_ptr[u + 1]; j += 32) {
+      const double r = (double)__ldg(R + __ldg(eid + j));
+      acc += WEIGHTED ? (double)__ldg(val + j) * r : r;
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) p[u] = (float)(1.0 - 0.5 * acc);
+  }
+}
+
+__global__ void k_edge_curvature(const int32_t* __restrict__ eu, const int32_t* __restrict__ ev,
+                                 const float* __restrict__ p, const float* __restrict__ R,
+                                 int64_t m, float* __restrict__ kappa) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < m;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const float s = p[eu[e]] + p[ev[e]];
+    kappa[e] = __fdiv_rn(2.f * s, R[e]);
+  }
+}
+
+// ---------------------------------------------------------------------------- sampling (§3.2)
+struct ProbWork {
+  double* qnode;     // [n]
+  float* part_min;   // [MAX_GRID]
+  float* part_max;   // [MAX_GRID]
+  double* part_qn;   // [MAX_GRID]
+  double* part_cnt;  // [MAX_GRID]
+  double* part_qe;   // [MAX_GRID]
+  double* scal;      // [0] kmin [1] kmax [2] sum qnode [3] #non-isolated [4] sum qedge
+};
+
+void plan_probs(Arena& a, ProbWork& w, int32_t n) {
+  w.qnode = a.take<double>(n);
+  w.part_min = a.take<float>(MAX_GRID);
+  w.part_max = a.take<float>(MAX_GRID);
+  w.part_qn = a.take<double>(MAX_GRID);
+  w.part_cnt = a.take<double>(MAX_GRID);
+  w.part_qe = a.take<double>(MAX_GRID);
+  w.scal = a.take<double>(8);
+}
+
+template <class V, class Op>
+__device__ __forceinline__ V block_reduce(V v, Op op, V* sh) {
+  sh[threadIdx.x] = v;
+  __syncthreads();
+  for (int s = blockDim.x / 2; s > 0; s >>= 1) {
+    if (threadIdx.x < s) sh[threadIdx.x] = op(sh[threadIdx.x], sh[threadIdx.x + s]);
+    __syncthreads();
+  }
+  V r = sh[0];
+  __syncthreads();
+  return r;
+}
+
+struct MinF {
+  __device__ float operator()(float a, float b) const { return fminf(a, b); }
+};
+struct MaxF {
+  __device__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
+struct AddD {
+  __device__ double operator()(double a, double b) const { return a + b; }
+};
+
+__global__ void __launch_bounds__(T)
+    k_kappa_minmax(const float* __restrict__ kappa, int64_t m, float* part_min, float* part_max) {
+  __shared__ float sh[T];
+  float lo = FLT_MAX, hi = -FLT_MAX;
+  for (int64_t e = (int64_t)blockIdx.x * T + threadIdx.x; e < m; e += (int64_t)gridDim.x * T) {
+    const float k = kappa[e];
+    lo = fminf(lo, k);
+    hi = fmaxf(hi, k);
+  }
+  lo = block_reduce(lo, MinF{}, sh);
+  hi = block_reduce(hi, MaxF{}, sh);
+  if (threadIdx.x == 0) {
+    part_min[blockIdx.x] = lo;
+    part_max[blockIdx.x] = hi;
+  }
+}
+
+__global__ void __launch_bounds__(T) k_minmax_final(const float* part_min, const float* part_max,
+                                                    int nparts, double* scal) {
+  __shared__ float sh[T];
+  float lo = FLT_MAX, hi = -FLT_MAX;
+  for (int i = threadIdx.x; i < nparts; i += T) {
+    lo = fminf(lo, part_min[i]);
+    hi = fmaxf(hi, part_max[i]);
+  }
+  lo = block_reduce(lo, MinF{}, sh);
+  hi = block_reduce(hi, MaxF{}, sh);
+  if (threadIdx.x == 0) {
+    scal[0] = lo;
+    scal[1] = hi;
+  }
+}
+
+// Eq. 7 row sums: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta)
+__global__ void __launch_bounds__(T)
+    k_qnode(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ eid,
+            const float* __restrict__ kappa, int32_t n, double eta, const double* scal,
+            double* __restrict__ qnode, double* part_qn, double* part_cnt) {
+  __shared__ double sh[T];
+  const int lane = threadIdx.x & 31;
+  const int64_t wpb = T / 32;
+  const double kmin = scal[0];
+  const double inv = 1.0 / (scal[1] - scal[0] + eta);
+  double tq = 0.0, tc = 0.0;
+  for (int64_t u = (int64_t)blockIdx.x * wpb + threadIdx.x / 32; u < n;
+       u += (int64_t)gridDim.x * wpb) {
+    const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
+    double acc = 0.0;
+    for (int64_t j = j0 + lane; j < j1; j += 32) acc += ((double)__ldg(kappa + __ldg(eid + j)) - kmin) * inv;
+    acc = warp_sum(acc);
+    if (lane == 0) {
+      qnode[u] = acc;
+      tq += acc;
+      tc += (j1 > j0) ? 1.0 : 0.0;
+    }
+  }
+  tq = block_reduce(tq, AddD{}, sh);
+  tc = block_reduce(tc, AddD{}, sh);
+  if (threadIdx.x == 0) {
+    part_qn[blockIdx.x] = tq;
+    part_cnt[blockIdx.x] = tc;
+  }
+}
+
+// Eq. 8: q_e = sqrt(max(-kappa_e + 2 kappa_max, 0)) + 1
+__device__ __forceinline__ float edge_weight(float k, float kmax) {
+  return sqrtf(fmaxf(-k + 2.f * kmax, 0.f)) + 1.f;
+}
+
+__global__ void __launch_bounds__(T)
+    k_qedge(const float* __restrict__ kappa, int64_t m, const double* scal, double* part_qe) {
+  __shared__ double sh[T];
+  const float kmax = (float)scal[1];
+  double acc = 0.0;
+  for (int64_t e = (int64_t)blockIdx.x * T + threadIdx.x; e < m; e += (int64_t)gridDim.x * T)
+    acc += (double)edge_weight(kappa[e], kmax);
+  acc = block_reduce(acc, AddD{}, sh);
+  if (threadIdx.x == 0) part_qe[blockIdx.x] = acc;
+}
+
+__global__ void __launch_bounds__(T) k_sums_final(const double* part_qn, const double* part_cnt,
+                                                  int np_node, const double* part_qe, int np_edge,
+                                                  double* scal) {
+  __shared__ double sh[T];
+  double a = 0.0, b = 0.0, c = 0.0;
+  for (int i = threadIdx.x; i < np_node; i += T) {
+    a += part_qn[i];
+    b += part_cnt[i];
+  }
+  for (int i = threadIdx.x; i < np_edge; i += T) c += part_qe[i];
+  a = block_reduce(a, AddD{}, sh);
+  b = block_reduce(b, AddD{}, sh);
+  c = block_reduce(c, AddD{}, sh);
+  if (threadIdx.x == 0) {
+    scal[2] = a;
+    scal[3] = b;
+    scal[4] = c;
+  }
+}
+
+__global__ void k_normalize(const int64_t* __restrict__ row_ptr, const double* __restrict__ qnode,
+                            int32_t n, const float* __restrict__ kappa, int64_t m,
+                            const double* scal, float* __restrict__ prob_node,
+                            float* __restrict__ prob_edge) {
+  const double tot_n = scal[2], cnt = scal[3], tot_e = scal[4];
+  const double inv_n = tot_n > 0.0 ? 1.0 / tot_n : 0.0;
+  const double uni = cnt > 0.0 ? 1.0 / cnt : 0.0;
+  const double inv_e = tot_e > 0.0 ? 1.0 / tot_e : 0.0;
+  const float kmax = (float)scal[1];
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n; u += stride) {
+    double pr;
+    if (tot_n > 0.0)
+      pr = qnode[u] * inv_n;
+    else  // every Eq. 7 weight vanished: uniform over the nodes with an edge
+      pr = row_ptr[u + 1] > row_ptr[u] ? uni : 0.0;
+    prob_node[u] = (float)pr;
+  }
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < m; e += stride)
+    prob_edge[e] = (float)((double)edge_weight(kappa[e], kmax) * inv_e);
+}
+
+}  // namespace
+}  // namespace erc
+
+using namespace erc;
+
+extern "C" erc_status erc_edge_resistance(const erc_graph* g, const float* X, int32_t ld,
+                                          int32_t kc, float* R_acc, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
+  ERC_REQUIRE(X && (reinterpret_cast<uintptr_t>(X) & 15) == 0, "X must be 16-byte aligned");
+  ERC_REQUIRE(R_acc || g->m == 0, "R_acc is required");
+  if (g->m == 0) return ERC_OK;
+  cudaStream_t s = as_stream(stream);
+  return dispatch_shape(ld / 4, [&](auto lpr, auto vpl) -> erc_status {
+    constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
+    const int64_t nseg = (g->m + 31) / 32;
+    k_edge_resistance<LPR, VPL><<<grid_for(nseg, T / LPR), T, 0, s>>>(g->eu, g->ev, g->m, X, ld,
+                                                                       kc, R_acc);
+    ERC_CUDA(cudaGetLastError());
+    return ERC_OK;
+  });
+}
+
+extern "C" erc_status erc_curvature(const erc_graph* g, const float* R, float* p_node,
+                                    float* kappa, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(p_node && (kappa || g->m == 0) && (R || g->m == 0), "R, p_node, kappa required");
+  cudaStream_t s = as_stream(stream);
+  if (g->val)
+    k_node_curvature<true><<<grid_for(g->n, T / 32), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
+                                                                R, g->n, p_node);
+  else
+    k_node_curvature<false><<<grid_for(g->n, T / 32), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
+                                                                 R, g->n, p_node);
+  ERC_CUDA(cudaGetLastError());
+  if (g->m > 0) {
+    k_edge_curvature<<<grid_for(g->m, T), T, 0, s>>>(g->eu, g->ev, p_node, R, g->m, kappa);
+    ERC_CUDA(cudaGetLastError());
+  }
+  return ERC_OK;
+}
+
+extern "C" size_t erc_sampling_probs_workspace_size(int32_t n, int64_t m) {
+  (void)m;
+  if (n < 1) return 0;
+  Arena a(nullptr);
+  ProbWork w;
+  plan_probs(a, w, n);
+  return a.used + 256;
+}
+
+extern "C" erc_status erc_sampling_probs(const erc_graph* g, const float* kappa, float eta,
+                                         float* prob_node, float* prob_edge, void* ws,
+                                         size_t ws_bytes, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(eta > 0.f && isfinite(eta), "eta must be positive");
+  ERC_REQUIRE(prob_node && ((kappa && prob_edge) || g->m == 0), "kappa and outputs required");
+  if (ws_bytes < erc_sampling_probs_workspace_size(g->n, g->m))
+    return set_error(ERC_ERR_CAPACITY, "workspace too small");
+  cudaStream_t s = as_stream(stream);
+  Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  ProbWork w;
+  plan_probs(ar, w, g->n);
+  if (g->m == 0) {
+    ERC_CUDA(cudaMemsetAsync(prob_node, 0, (size_t)g->n * sizeof(float), s));
+    return ERC_OK;
+  }
+  const int ge = grid_for(g->m, T);
+  k_kappa_minmax<<<ge, T, 0, s>>>(kappa, g->m, w.part_min, w.part_max);
+  ERC_CUDA(cudaGetLastError());
+  k_minmax_final<<<1, T, 0, s>>>(w.part_min, w.part_max, ge, w.scal);
+  ERC_CUDA(cudaGetLastError());
+  const int gn = grid_for(g->n, T / 32);
+  k_qnode<<<gn, T, 0, s>>>(g->row_ptr, g->csr_eid, kappa, g->n, (double)eta, w.scal, w.qnode,
+                           w.part_qn, w.part_cnt);
+  ERC_CUDA(cudaGetLastError());
+  k_qedge<<<ge, T, 0, s>>>(kappa, g->m, w.scal, w.part_qe);
+  ERC_CUDA(cudaGetLastError());
+  k_sums_final<<<1, T, 0, s>>>(w.part_qn, w.part_cnt, gn, w.part_qe, ge, w.scal);
+  ERC_CUDA(cudaGetLastError());
+  k_normalize<<<grid_for(g->n > g->m ? g->n : g->m, T), T, 0, s>>>(
+      g->row_ptr, w.qnode, g->n, kappa, g->m, w.scal, prob_node, prob_edge);
+  ERC_CUDA(cudaGetLastError());
+  return ERC_OK;
+}

@@ -1,0 +1,210 @@
+// erc_internal.cuh -- shared internals of liberc.so (not part of the public ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <cstddef>
+#include <type_traits>
+#include <utility>
+
+#include "../../include/erc.h"
+
+namespace erc {
+
+// ------------------------------------------------------------------------------------------------
+// host-side errors
+// ------------------------------------------------------------------------------------------------
+erc_status set_error(erc_status code, const char* fmt, ...);
+void clear_error();
+
+#define ERC_CUDA(call)                                                                    \
+  do {                                                                                    \
+    cudaError_t e_ = (call);                                                              \
+    if (e_ != cudaSuccess)                                                                \
+      return ::erc::set_error(ERC_ERR_CUDA, "%s:%d %s: %s", __FILE__, __LINE__, #call,      \
+                              cudaGetErrorString(e_));                                    \
+  } while (0)
+
+#define ERC_TRY(expr)                   \
+  do {                                  \
+    erc_status st_ = (expr);            \
+    if (st_ != ERC_OK) return st_;      \
+  } while (0)
+
+#define ERC_REQUIRE(cond, ...)                                          \
+  do {                                                                  \
+    if (!(cond)) return ::erc::set_error(ERC_ERR_INVALID_ARG, __VA_ARGS__); \
+  } while (0)
+
+inline cudaStream_t as_stream(erc_stream s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// SM count of the current device (cached per device).
+int sm_count();
+
+// ------------------------------------------------------------------------------------------------
+// workspace carving: the same plan runs once to size (base == nullptr) and once to carve
+// ------------------------------------------------------------------------------------------------
+struct Arena {
+  char* base;
+  size_t used = 0;
+  explicit Arena(void* b) : base(static_cast<char*>(b)) {}
+  template <class T>
+  T* take(size_t count) {
+    used = (used + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + used) : nullptr;
+    used += count * sizeof(T);
+    return p;
+  }
+};
+
+// ------------------------------------------------------------------------------------------------
+// double-float ("float2" hi + lo) accumulation: error-free transformations on float32 units.
+// GB300 runs float64 at a small fraction of its float32 rate, so long dot products are kept in a
+// float pair (about 44 significant bits) and only the final per-column values go to float64.
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ float2 df_two_sum(float a, float b) {
+  float s = __fadd_rn(a, b);
+  float bb = __fsub_rn(s, a);
+  float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return make_float2(s, e);
+}
+__device__ __forceinline__ float2 df_norm(float hi, float e) {
+  float h = __fadd_rn(hi, e);
+  return make_float2(h, __fsub_rn(e, __fsub_rn(h, hi)));
+}
+__device__ __forceinline__ float2 df_add(float2 a, float2 b) {
+  float2 s = df_two_sum(a.x, b.x);
+  return df_norm(s.x, __fadd_rn(s.y, __fadd_rn(a.y, b.y)));
+}
+// acc + a*b with the product kept exact (a*b = p + pe)
+__device__ __forceinline__ float2 df_fma(float2 acc, float a, float b) {
+  float p = __fmul_rn(a, b);
+  float pe = __fmaf_rn(a, b, -p);
+  float2 s = df_two_sum(acc.x, p);
+  return df_norm(s.x, __fadd_rn(s.y, __fadd_rn(acc.y, pe)));
+}
+__device__ __forceinline__ double df_value(float2 a) { return (double)a.x + (double)a.y; }
+
+// ------------------------------------------------------------------------------------------------
+// deterministic grid-wide per-column reduction of float2 partials.
+// Blocks publish their partial row; the last block of each group of RED_GROUP blocks sums the
+// group in block order, and the last group-finisher sums the group rows in group order.  The
+// result does not depend on which block arrives when.  Counters must be zero at kernel start; the
+// finishers reset them, so consecutive launches on one stream can share the buffers.
+// ------------------------------------------------------------------------------------------------
+constexpr int RED_GROUP = 32;
+constexpr int MAX_GRID = 8192;  // the largest grid any reducing kernel launches
+
+struct ColReduce {
+  float2* part1;  // [MAX_GRID][ld]
+  float2* part2;  // [MAX_GRID / RED_GROUP][ld]
+  unsigned* cnt;  // [MAX_GRID / RED_GROUP + 1]
+};
+
+inline void plan_colreduce(Arena& a, ColReduce& cr, int ld) {
+  cr.part1 = a.take<float2>((size_t)MAX_GRID * ld);
+  cr.part2 = a.take<float2>((size_t)(MAX_GRID / RED_GROUP) * ld);
+  cr.cnt = a.take<unsigned>(MAX_GRID / RED_GROUP + 1);
+}
+inline size_t colreduce_counter_bytes() { return sizeof(unsigned) * (MAX_GRID / RED_GROUP + 1); }
+
+// All threads of every block call this once `bpart` (shared, ld entries) holds the block's
+// partial.  Returns true in exactly one block, whose `res` (shared, ld entries) then holds the
+// totals.
+__device__ __forceinline__ bool grid_colreduce(const ColReduce& cr, const float2* bpart,
+                                               float2* res, int ld) {
+  __shared__ int s_last;
+  const int G = gridDim.x, b = blockIdx.x;
+  const int grp = b / RED_GROUP;
+  const int ng = (G + RED_GROUP - 1) / RED_GROUP;
+  const int gsize = min(RED_GROUP, G - grp * RED_GROUP);
+  for (int c = threadIdx.x; c < ld; c += blockDim.x) cr.part1[(size_t)b * ld + c] = bpart[c];
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&cr.cnt[grp], 1u) == (unsigned)(gsize - 1));
+  __syncthreads();
+  if (!s_last) return false;
+  __threadfence();
+  for (int c = threadIdx.x; c < ld; c += blockDim.x) {
+    float2 acc = make_float2(0.f, 0.f);
+    const float2* src = cr.part1 + (size_t)grp * RED_GROUP * ld + c;
+    for (int k = 0; k < gsize; ++k) acc = df_add(acc, __ldcg(src + (size_t)k * ld));
+    cr.part2[(size_t)grp * ld + c] = acc;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    cr.cnt[grp] = 0;
+    s_last = (atomicAdd(&cr.cnt[ng], 1u) == (unsigned)(ng - 1));
+  }
+  __syncthreads();
+  if (!s_last) return false;
+  __threadfence();
+  for (int c = threadIdx.x; c < ld; c += blockDim.x) {
+    float2 acc = make_float2(0.f, 0.f);
+    for (int k = 0; k < ng; ++k) acc = df_add(acc, __ldcg(cr.part2 + (size_t)k * ld + c));
+    res[c] = acc;
+  }
+  if (threadIdx.x == 0) cr.cnt[ng] = 0;
+  __syncthreads();
+  return true;
+}
+
+// ------------------------------------------------------------------------------------------------
+// row-block shapes: a row of ld floats is nvec = ld/4 float4s, handled by a group of LPR lanes
+// with VPL float4s per lane (LPR * VPL >= nvec).
+// ------------------------------------------------------------------------------------------------
+template <int V>
+using ic = std::integral_constant<int, V>;
+
+template <class F>
+inline erc_status dispatch_shape(int nvec, F&& f) {
+  if (nvec <= 4) return f(ic<4>{}, ic<1>{});
+  if (nvec <= 8) return f(ic<8>{}, ic<1>{});
+  if (nvec <= 16) return f(ic<16>{}, ic<1>{});
+  if (nvec <= 32) return f(ic<32>{}, ic<1>{});
+  if (nvec <= 64) return f(ic<32>{}, ic<2>{});
+  if (nvec <= 128) return f(ic<32>{}, ic<4>{});
+  if (nvec <= 256) return f(ic<32>{}, ic<8>{});
+  return set_error(ERC_ERR_INVALID_ARG, "ld > 1024 is not supported");
+}
+
+constexpr int MAX_LD = 1024;
+
+template <int LPR>
+__device__ __forceinline__ unsigned group_mask() {
+  if constexpr (LPR == 32) {
+    return 0xffffffffu;
+  } else {
+    const unsigned lane = threadIdx.x & 31u;
+    return ((1u << LPR) - 1u) << (lane & ~(unsigned)(LPR - 1));
+  }
+}
+
+// grid size for a grid-stride kernel: at most `waves` resident waves of blocks, at least 1
+inline int grid_for(long long work_items, int items_per_block, int waves_blocks_per_sm = 8) {
+  long long g = (work_items + items_per_block - 1) / items_per_block;
+  long long cap = (long long)sm_count() * waves_blocks_per_sm;
+  if (g > cap) g = cap;
+  if (g > MAX_GRID) g = MAX_GRID;
+  if (g < 1) g = 1;
+  return (int)g;
+}
+
+// ------------------------------------------------------------------------------------------------
+// internal entry points shared between translation units
+// ------------------------------------------------------------------------------------------------
+erc_status check_graph(const erc_graph* g);
+size_t scan_temp_bytes(int64_t n);
+// exclusive scan of int64 `in` (or of the 0/1 flags in `flags` when `in` is null) into `out`;
+// `total` (device, may be null) receives the sum.
+erc_status exclusive_scan_i64(const int64_t* in, const uint8_t* flags, int64_t* out, int64_t n,
+                              int64_t* total, void* tmp, cudaStream_t s);
+size_t radix_sort_temp_bytes(int64_t n);
+// stable LSD radix sort of (key, value) pairs on the low `bits` key bits; the result is in
+// keys/vals (the *_alt buffers are scratch of the same size)
+erc_status radix_sort_pairs(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
+                            int64_t n, int bits, void* tmp, cudaStream_t s);
+
+}  // namespace erc

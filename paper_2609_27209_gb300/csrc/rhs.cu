@@ -1,0 +1,149 @@
+// rhs.cu -- erc_jl_rhs: Y = B^T W^{1/2} Q for a batch of projection columns (§3.1.2), with the
+// signs of Q generated in registers by Philox4x32-10 and never stored.
+//
+// Row u of Y gathers over u's CSR slots: the canonical edge e = (eu, ev) contributes
+// sigma * sqrt(w_e) * Q[e, c] with sigma = +1 when u = eu (the smaller id) and -1 otherwise.
+// Summing in CSR order makes Y deterministic without atomics.
+#include "erc_internal.cuh"
+
+namespace erc {
+namespace {
+
+// Philox4x32-10 block function (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64
+// multiplies, with the key bumped by the Weyl constants between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+    k.x += 0x9E3779B9u;
+    k.y += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// the 32-bit Philox word holding the sign bits of columns 32*(c/32) .. +31 of edge e
+__device__ __forceinline__ uint32_t sign_word(uint2 key, uint32_t e, int c, int& cached_g,
+                                              uint4& cached) {
+  const int g = c >> 7;
+  if (g != cached_g) {
+    cached = philox4x32_10(make_uint4((uint32_t)g, 0u, e, 0u), key);
+    cached_g = g;
+  }
+  const int wi = (c >> 5) & 3;
+  return wi == 0 ? cached.x : wi == 1 ? cached.y : wi == 2 ? cached.z : cached.w;
+}
+
+template <int LPR, int VPL, bool WEIGHTED>
+__global__ void __launch_bounds__(256)
+    k_jl_rhs(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ col,
+             const float* __restrict__ val, const int32_t* __restrict__ csr_eid, int32_t n,
+             uint2 key, float inv_sqrt_k, int32_t c0, int32_t kc, int32_t ld, float* __restrict__ Y) {
+  const int gl = threadIdx.x & (LPR - 1);
+  const int groups_per_block = blockDim.x / LPR;
+  const int64_t ngroups = (int64_t)gridDim.x * groups_per_block;
+  const int nvec = ld >> 2;
+  for (int64_t u = (int64_t)blockIdx.x * groups_per_block + threadIdx.x / LPR; u < n;
+       u += ngroups) {
+    float4 acc[VPL];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
+    for (int64_t j = j0; j < j1; ++j) {
+      const int32_t nb = col[j];
+      const uint32_t e = (uint32_t)csr_eid[j];
+      float coef = WEIGHTED ? sqrtf(val[j]) * inv_sqrt_k : inv_sqrt_k;
+      if (nb < u) coef = -coef;  // u is the larger endpoint: row e of B is e_nb - e_u
+      int cg = -1;
+      uint4 cw;
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q < nvec && 4 * q < kc) {
+          const int c = c0 + 4 * q;  // c0 % 4 == 0: the four columns share one word
+          const uint32_t bits = sign_word(key, e, c, cg, cw) >> (c & 31);
+          acc[v].x += (bits & 1u) ? -coef : coef;
+          acc[v].y += (bits & 2u) ? -coef : coef;
+          acc[v].z += (bits & 4u) ? -coef : coef;
+          acc[v].w += (bits & 8u) ? -coef : coef;
+        }
+      }
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q < nvec) {
+        float4 o = acc[v];
+        const int cb = 4 * q;
+        if (cb + 0 >= kc) o.x = 0.f;
+        if (cb + 1 >= kc) o.y = 0.f;
+        if (cb + 2 >= kc) o.z = 0.f;
+        if (cb + 3 >= kc) o.w = 0.f;
+        reinterpret_cast<float4*>(Y + (size_t)u * ld)[q] = o;
+      }
+    }
+  }
+}
+
+__global__ void k_philox_signs(uint2 key, int64_t e0, int64_t e1, int32_t c0, int32_t c1,
+                               uint32_t* __restrict__ out) {
+  const int64_t ncol = c1 - c0;
+  const int64_t total = (e1 - e0) * ncol;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t e = e0 + t / ncol;
+    const int c = c0 + (int)(t % ncol);
+    const uint4 w = philox4x32_10(
+        make_uint4((uint32_t)(c >> 7), 0u, (uint32_t)(e & 0xffffffff), (uint32_t)(e >> 32)), key);
+    const int wi = (c >> 5) & 3;
+    const uint32_t word = wi == 0 ? w.x : wi == 1 ? w.y : wi == 2 ? w.z : w.w;
+    out[t] = (word >> (c & 31)) & 1u;
+  }
+}
+
+}  // namespace
+}  // namespace erc
+
+using namespace erc;
+
+extern "C" erc_status erc_jl_rhs(const erc_graph* g, uint64_t seed, int32_t K, int32_t c0,
+                                 int32_t kc, float* Y, int32_t ld, erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  ERC_REQUIRE(K >= 1 && kc >= 1 && c0 >= 0 && (int64_t)c0 + kc <= K,
+              "need 0 <= c0, 1 <= kc, c0 + kc <= K (c0=%d kc=%d K=%d)", c0, kc, K);
+  ERC_REQUIRE(c0 % 4 == 0, "c0 must be a multiple of 4 (got %d)", c0);
+  ERC_REQUIRE(ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad ld %d for kc %d", ld, kc);
+  ERC_REQUIRE(Y && (reinterpret_cast<uintptr_t>(Y) & 15) == 0, "Y must be 16-byte aligned");
+  ERC_REQUIRE(g->m < (int64_t(1) << 31), "m must be < 2^31");
+  cudaStream_t s = as_stream(stream);
+  const uint2 key = make_uint2((uint32_t)(seed & 0xffffffffu), (uint32_t)(seed >> 32));
+  const float inv_sqrt_k = (float)(1.0 / sqrt((double)K));
+  return dispatch_shape(ld / 4, [&](auto lpr, auto vpl) -> erc_status {
+    constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
+    const int grid = grid_for(g->n, 256 / LPR);
+    if (g->val)
+      k_jl_rhs<LPR, VPL, true><<<grid, 256, 0, s>>>(g->row_ptr, g->col, g->val, g->csr_eid, g->n,
+                                                    key, inv_sqrt_k, c0, kc, ld, Y);
+    else
+      k_jl_rhs<LPR, VPL, false><<<grid, 256, 0, s>>>(g->row_ptr, g->col, g->val, g->csr_eid, g->n,
+                                                     key, inv_sqrt_k, c0, kc, ld, Y);
+    ERC_CUDA(cudaGetLastError());
+    return ERC_OK;
+  });
+}
+
+extern "C" erc_status erc_philox_signs(uint64_t seed, int64_t e0, int64_t e1, int32_t c0,
+                                       int32_t c1, uint32_t* out_bits, erc_stream stream) {
+  clear_error();
+  ERC_REQUIRE(e0 >= 0 && e1 >= e0 && c0 >= 0 && c1 >= c0, "bad ranges");
+  ERC_REQUIRE(out_bits || e1 == e0 || c1 == c0, "out_bits is required");
+  const int64_t total = (e1 - e0) * (int64_t)(c1 - c0);
+  if (total == 0) return ERC_OK;
+  const uint2 key = make_uint2((uint32_t)(seed & 0xffffffffu), (uint32_t)(seed >> 32));
+  k_philox_signs<<<grid_for(total, 256), 256, 0, as_stream(stream)>>>(key, e0, e1, c0, c1,
+                                                                      out_bits);
+  ERC_CUDA(cudaGetLastError());
+  return ERC_OK;
+}

@@ -243,3 +243,23 @@ def random_connected(n, extra, seed, weighted=True):
                                                  rng.integers(0, n, extra), n)])
     keys = keys[(keys // n) != (keys % n)]
     return _finish(rng, n, keys, "uniform_0.5_2" if weighted else "unit")
+
+
+# ----------------------------------------------------------------------------------------------
+# seeded dense inputs for single-call parity tests
+# ----------------------------------------------------------------------------------------------
+def random_block(n, kc, ld, seed):
+    """n x ld float32 block: standard normal in the first kc columns, zero padding after."""
+    rng = np.random.default_rng(seed)
+    X = np.zeros((n, ld), np.float32)
+    X[:, :kc] = rng.standard_normal((n, kc)).astype(np.float32)
+    return X
+
+
+def random_positive(size, seed, lo=0.05, hi=2.0):
+    """float32 values uniform in [lo, hi)."""
+    return np.random.default_rng(seed).uniform(lo, hi, size).astype(np.float32)
+
+
+def random_normal(size, seed, scale=1.0):
+    return (np.random.default_rng(seed).standard_normal(size) * scale).astype(np.float32)

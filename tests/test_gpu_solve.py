@@ -1,0 +1,131 @@
+"""GPU parity of the CG solve (§3.1.3) and of the whole path (Algorithm 1 + §3.2) with the oracle.
+
+Tolerances: R_hat per edge max relative error 1e-3 and median 1e-5; kappa absolute error at
+most 1e-3 * max|kappa| (against the fp64 oracle run with the same graph, seed, eps and tau).
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import erc_oracle as O
+from paper_2609_27209_gb300 import erc, synth
+
+from ._gpu import build_both, dev, host, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _check_R(R, Rr, max_rel=1e-3, med_rel=1e-5):
+    rel = np.abs(R.astype(np.float64) - Rr) / Rr
+    assert rel.max() <= max_rel and np.median(rel) <= med_rel, (rel.max(), np.median(rel))
+    return rel
+
+
+def _check_kappa(k, kr):
+    err = np.abs(k.astype(np.float64) - kr)
+    assert err.max() <= 1e-3 * np.abs(kr).max(), (err.max(), np.abs(kr).max())
+
+
+@pytest.mark.parametrize("kc", [8, 64])
+def test_cg_matches_oracle_cg(kc):
+    n, src, dst, w = synth.random_connected(3000, 12000, seed=4)
+    g, ref = build_both(n, src, dst, w)
+    K, eps, tol = 64, 1e-3, 1e-6
+    Y = erc.erc_jl_rhs(g, 5, K, 0, kc)
+    X, iters, relres, st = erc.erc_batched_cg(g, eps, Y, kc, tol)
+    assert st == erc.ERC_OK
+    Yr = O.jl_rhs(ref, 5, K, 0, kc)
+    Xr, itr, rrr, ok = O.batched_cg(ref, eps, Yr, tol)
+    Rg = torch.zeros(g.m, device=dev())
+    erc.erc_edge_resistance(g, X, kc, Rg)
+    _check_R(host(Rg), O.edge_resistance(ref, Xr))
+    it = host(iters)
+    assert np.all(np.abs(it - itr) <= 0.1 * itr + 2), (it, itr)
+    assert np.all(host(relres) <= 2 * tol), host(relres)
+    assert np.all(host(X)[:, kc:] == 0)
+
+
+def test_cg_not_converged_and_zero_columns():
+    n, src, dst, w = synth.random_connected(1000, 3000, seed=5)
+    g, ref = build_both(n, src, dst, w)
+    Y = erc.erc_jl_rhs(g, 5, 16, 0, 16)
+    Y[:, 3] = 0
+    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, 16, 1e-6, max_iter=3)
+    assert st == erc.ERC_ERR_NOT_CONVERGED
+    it = host(iters)
+    assert it[3] == 0 and np.all(np.delete(it, 3) == 3)
+    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, 16, 1e-6)
+    assert st == erc.ERC_OK and host(iters)[3] == 0 and float(host(relres)[3]) == 0.0
+    assert torch.all(X[:, 3] == 0)
+
+
+def test_cg_rejects_bad_arguments():
+    n, src, dst, w = synth.random_connected(100, 300, seed=6)
+    g, _ = build_both(n, src, dst, w)
+    Y = erc.erc_jl_rhs(g, 5, 8, 0, 8)
+    for kw in [dict(eps=0.0), dict(eps=-1.0), dict(tol=float("nan"))]:
+        a = dict(eps=1e-3, tol=1e-6)
+        a.update(kw)
+        with pytest.raises(erc.ErcError) as e:
+            erc.erc_batched_cg(g, a["eps"], Y, 8, a["tol"])
+        assert e.value.status == erc.ERC_ERR_INVALID_ARG
+
+
+def _run_both(name, K=None, kc=None, columns=None):
+    wl = synth.WORKLOADS[name]
+    n, src, dst, w = synth.make_graph(name)
+    K = K or wl.K[0]
+    kc = kc or wl.kc
+    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
+    out = erc.erc_run(n, to_dev(src), to_dev(dst), to_dev(w), prm)
+    ref = O.erc_lg(n, src, dst, w, K, kc, wl.eps, wl.tol, synth.JL_SEED)
+    return (n, src, dst, w), prm, out, ref
+
+
+@pytest.mark.parametrize("name", ["ring_chords_n2000", "sbm_n20000"])
+def test_pipeline_matches_oracle(name):
+    inp, prm, out, ref = _run_both(name)
+    assert out["status"] == erc.ERC_OK
+    g = ref["graph"]
+    assert out["m"] == g["m"]
+    np.testing.assert_array_equal(host(out["eu"]), g["eu"])
+    np.testing.assert_array_equal(host(out["ev"]), g["ev"])
+    _check_R(host(out["R"]), ref["R"])
+    _check_kappa(host(out["kappa"]), ref["kappa"])
+    np.testing.assert_allclose(host(out["p"]), ref["p"], atol=1e-3 * np.abs(ref["p"]).max())
+    np.testing.assert_allclose(host(out["prob_edge"]), ref["prob_edge"], rtol=1e-3)
+    np.testing.assert_allclose(host(out["prob_node"]), ref["prob_node"], rtol=1e-2,
+                               atol=1e-3 * ref["prob_node"].max())
+    assert abs(float(out["prob_node"].double().sum()) - 1) < 1e-5
+    assert abs(float(out["prob_edge"].double().sum()) - 1) < 1e-5
+    assert np.all(host(out["relres"]) <= 2 * prm.tol)
+
+
+def test_pipeline_host_path_and_determinism():
+    name = "ring_chords_n2000"
+    wl = synth.WORKLOADS[name]
+    n, src, dst, w = synth.make_graph(name)
+    prm = erc.Params(K=wl.K[0], kc=32, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
+    a = erc.erc_run(n, to_dev(src), to_dev(dst), None, prm)
+    b = erc.erc_run(n, to_dev(src), to_dev(dst), None, prm)
+    h = erc.erc_run_host(n, torch.from_numpy(src).pin_memory(), torch.from_numpy(dst).pin_memory(),
+                         None, prm)
+    for k in ["eu", "ev", "R", "p", "kappa", "prob_node", "prob_edge", "iters", "relres"]:
+        assert torch.equal(a[k], b[k]), k
+        assert torch.equal(a[k].cpu(), h[k]), k
+
+
+def test_pipeline_batches_sum_to_whole():
+    """Streaming K in batches (Algorithm 1) gives the sum of per-batch contributions."""
+    name = "ring_chords_n2000"
+    wl = synth.WORKLOADS[name]
+    n, src, dst, w = synth.make_graph(name)
+    g, ref = build_both(n, src, dst, w)
+    R = torch.zeros(g.m, device=dev())
+    for c0 in (0, 32):
+        Y = erc.erc_jl_rhs(g, synth.JL_SEED, 64, c0, 32)
+        X, _, _, st = erc.erc_batched_cg(g, wl.eps, Y, 32, wl.tol)
+        erc.erc_edge_resistance(g, X, 32, R)
+    full = erc.erc_run(n, to_dev(src), to_dev(dst), None,
+                       erc.Params(K=64, kc=64, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED))
+    np.testing.assert_allclose(host(R), host(full["R"]), rtol=1e-4)
