@@ -1,0 +1,361 @@
+#!/usr/bin/env python
+"""ERC-LG curvature throughput on GB300.
+
+One step = the whole path on one synthetic graph with its inputs resident in HBM: Laplacian build,
+then for every batch of projection columns the Philox right-hand sides, the column-wise CG solve
+and the edge-resistance accumulation, then curvature (Eq. 2) and the sampling probabilities
+(Eq. 7-8).  The metric is curvature edges per second (m / step time); the JSON line also carries
+the end-to-end number through the host-memory C-ABI call, the roofline of the dominant kernel
+(the L_eps P gather), the CPU oracle as a reported baseline, clocks and the kernel-launch count.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config NAME]
+Under torchrun (N > 1) every rank owns K projection columns of a K*N projection (weak scaling)
+and the per-rank edge accumulators are summed with one all-reduce (Algorithm 1).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ERC-LG curvature edges/s end-to-end; CG SpMM HBM GB/s vs GB300 peak"
+DEFAULT_CONFIG = "sbm_n20000"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--K", type=int, default=None, help="projection dimension (per rank)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--spmm-reps", type=int, default=50)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------------------------ helpers
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                rows.append(f)
+        os.unlink(self.path)
+        if not rows:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d.get("hbm_gbs"), "measured"
+    return 6800.0, "fallback"
+
+
+def spmm_traffic(workload):
+    """DRAM bytes per launch of the gather kernel from a committed ncu summary, if still current."""
+    p = os.path.join(ROOT, "profiles", "spmm_traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p))
+    src = os.path.join(ROOT, "paper_2609_27209_gb300", "csrc", "cg.cu")
+    sha = hashlib.sha1(open(src, "rb").read()).hexdigest()
+    e = d.get(workload)
+    if not e or e.get("cg_cu_sha1") != sha:
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def spmm_algorithmic_bytes(n, m, kc, weighted):
+    """Bytes the operator must move once: CSR (col, weights, row_ptr) + read P + write AP."""
+    return 4 * 2 * m + (4 * 2 * m if weighted else 0) + 8 * (n + 1) + 2 * 4 * n * kc
+
+
+# ------------------------------------------------------------------------------------ oracle leg
+def oracle_sample(name, K, cols):
+    """Time the CPU oracle on the full graph with `cols` of the K projection columns and
+    extrapolate the column-proportional part to K.  Returns (edges/s, seconds, description)."""
+    import numpy as np
+
+    from oracle import erc_oracle as O
+    from paper_2609_27209_gb300 import synth
+
+    wl = synth.WORKLOADS[name]
+    n, src, dst, w = synth.make_graph(name)
+    t0 = time.perf_counter()
+    g = O.build_laplacian(n, src, dst, w)
+    t1 = time.perf_counter()
+    Y = O.jl_rhs(g, synth.JL_SEED, K, 0, cols)
+    X, it, _, _ = O.batched_cg(g, wl.eps, Y, wl.tol)
+    R = O.edge_resistance(g, X)
+    t2 = time.perf_counter()
+    p, kappa = O.curvature(g, R * (K / cols))
+    O.sampling_probs(g, kappa)
+    t3 = time.perf_counter()
+    est = (t1 - t0) + (t2 - t1) * (K / cols) + (t3 - t2)
+    desc = (f"full graph (n={n}, m={g['m']}), {cols} of {K} projection columns; build and "
+            f"curvature/probability tail timed once, the per-column solve scaled by {K}/{cols}")
+    return g["m"] / est, t3 - t0, desc, est
+
+
+def cpu_cores_used():
+    return 1  # numpy elementwise and scipy sparse products run single-threaded here
+
+
+# ------------------------------------------------------------------------------------ main legs
+def run_reference(args, world, rank):
+    from paper_2609_27209_gb300 import synth
+
+    wl = synth.WORKLOADS[args.config]
+    K = args.K or wl.K[0]
+    cols = max(4, K // 8)
+    if rank != 0:
+        return
+    for _ in range(args.warmup):
+        oracle_sample(args.config, K, cols)
+    vals, ests = [], []
+    for _ in range(args.steps):
+        v, _, desc, est = oracle_sample(args.config, K, cols)
+        vals.append(v)
+        ests.append(est)
+    value = len(vals) / sum(1.0 / v for v in vals)  # harmonic mean = m / mean time
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "edges/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * statistics.mean(ests), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.config, "K": K, "kc": wl.kc, "eps": wl.eps,
+                       "tol": wl.tol},
+            "cpu_baseline": {"value": value, "unit": "edges/s", "cores": cpu_cores_used(),
+                             "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": "edges/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, world, rank, local_rank):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_27209_gb300 import dist as edist
+    from paper_2609_27209_gb300 import erc, synth
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    wl = synth.WORKLOADS[args.config]
+    K = args.K or wl.K[0]
+    kc = min(wl.kc, K)
+    n, src, dst, w = synth.make_graph(args.config)
+    m_in = src.size
+    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
+    src_d = torch.from_numpy(src).to(dev)
+    dst_d = torch.from_numpy(dst).to(dev)
+    w_d = None if w is None else torch.from_numpy(w).to(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB of L2
+
+    if world == 1:
+        ws = erc.erc_run_workspace(n, m_in, prm, dev)
+        out = erc._run_outputs(n, m_in, K, dev)
+
+        def step():
+            return erc.erc_run(n, src_d, dst_d, w_d, prm, ws=ws, out=out)
+    else:
+        def allreduce(t):
+            dist.all_reduce(t, op=dist.ReduceOp.SUM)
+            return t
+
+        def step():
+            return edist.run_sharded(n, src_d, dst_d, w_d, prm, world, rank, allreduce)
+
+    res = None
+    for _ in range(args.warmup):
+        res = step()
+    torch.cuda.synchronize()
+    m = int(res["m"])
+    stream = torch.cuda.current_stream()
+    sampler = ClockSampler(local_rank)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = erc.erc_kernel_launches()
+    sampler.start()
+    times = []
+    for _ in range(args.steps):
+        flush.fill_(1)  # evict L2 between timed steps (outside the timed interval)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        res = step()
+        b.record(stream)
+        b.synchronize()
+        times.append(a.elapsed_time(b))
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    launches = erc.erc_kernel_launches() - launches0
+    if world > 1:
+        dist.barrier()
+    ms = statistics.mean(times)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    value = world * m / (ms_max / 1000.0)
+    iters = res.get("iters")
+    it = iters.float() if iters is not None else None
+
+    # ---- end to end through the host-memory C-ABI call (copies inside the timed region)
+    e2e = None
+    if not args.no_e2e and world == 1:
+        src_h = torch.from_numpy(src).pin_memory()
+        dst_h = torch.from_numpy(dst).pin_memory()
+        w_h = None if w is None else torch.from_numpy(w).pin_memory()
+        hws = erc.erc_run_host_workspace(n, m_in, prm, dev)
+        hout = erc._run_outputs(n, m_in, K, None, pin=True)
+        for _ in range(2):
+            erc.erc_run_host(n, src_h, dst_h, w_h, prm, ws=hws, out=hout)
+        et = []
+        for _ in range(max(3, args.steps // 2)):
+            flush.fill_(1)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            erc.erc_run_host(n, src_h, dst_h, w_h, prm, ws=hws, out=hout)
+            torch.cuda.synchronize()
+            et.append(time.perf_counter() - t0)
+        h2d = m_in * 4 * (2 if w is None else 3)
+        d2h = 5 * 4 * m + 2 * 4 * n + 2 * 4 * K
+        e2e = {"value": m / statistics.mean(et), "unit": "edges/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": 1000 * statistics.mean(et)}
+
+    # ---- roofline of the dominant kernel: the L_eps P gather (k_spmm), timed alone on the
+    # stream it is launched on, back to back as inside the CG loop
+    roof = None
+    if rank == 0:
+        g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
+        P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
+        for _ in range(5):
+            erc.erc_laplacian_apply(g, prm.eps, P, kc, want_pap=True)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.spmm_reps):
+            erc.erc_laplacian_apply(g, prm.eps, P, kc, want_pap=True)
+        b.record(stream)
+        b.synchronize()
+        t_spmm = a.elapsed_time(b) / args.spmm_reps / 1000.0
+        algo = spmm_algorithmic_bytes(n, g.m, kc, not g.unit_weights)
+        peak, src_kind = measured_peaks()
+        ach = algo / t_spmm / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+                "frac": ach / peak, "traffic": spmm_traffic(args.config),
+                "kernel": "k_spmm (L_eps P + p.Ap)", "algorithmic_bytes": algo,
+                "launch_us": t_spmm * 1e6, "peak_source": src_kind}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        # size the sample to roughly 15 s of CPU work from a 4-column probe
+        _, _, _, est4 = oracle_sample(args.config, K, 4)
+        per_col = est4 / K  # the probe's estimate is for all K columns
+        cols = int(min(K, max(4, (15.0 / max(per_col, 1e-9)) // 4 * 4)))
+        v, secs, desc, est = oracle_sample(args.config, K, cols)
+        cpu = {"value": v, "unit": "edges/s", "cores": cpu_cores_used(), "kind": "oracle",
+               "sample": desc, "seconds": secs}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "edges/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic",
+                "config": {"workload": args.config, "n": n, "m": m, "K": K, "kc": kc,
+                           "eps": wl.eps, "tol": wl.tol,
+                           "l2": "flushed (256 MiB write) before every timed step",
+                           "parallelism": f"projection columns over {world} rank(s)"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "clocks": clocks,
+                "cg_iters": None if it is None else {"mean": float(it.mean()),
+                                                     "max": float(it.max())}}
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, world, rank, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -77,6 +77,9 @@ typedef struct erc_params {
 
 const char* erc_version(void);
 const char* erc_last_error(void);
+/* Number of CUDA kernels this library has launched in this process so far (a CUDA-graph launch
+ * counts the kernels it contains).  For instrumentation only. */
+uint64_t erc_kernel_launches(void);
 
 /* ---------------------------------------------------------------------------------------------
  * erc_build_laplacian -- the simple undirected graph behind L = D - A = B^T W B (§3.1.1).

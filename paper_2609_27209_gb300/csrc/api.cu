@@ -1,6 +1,7 @@
 // api.cu -- error reporting, graph checks and the whole-path drivers erc_run / erc_run_host
 // (Algorithm 1 followed by §3.2), which stream the K projection columns in batches of kc so the
 // n x K embedding is never held.
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -12,7 +13,14 @@ namespace erc {
 
 namespace {
 thread_local char g_err[512] = "";
+thread_local bool g_capturing = false;
+std::atomic<unsigned long long> g_launches{0};
 }
+
+void count_launches(long long k) {
+  if (!g_capturing) g_launches.fetch_add((unsigned long long)k, std::memory_order_relaxed);
+}
+void set_capturing(bool on) { g_capturing = on; }
 
 erc_status set_error(erc_status code, const char* fmt, ...) {
   va_list ap;
@@ -105,6 +113,7 @@ erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, cons
   if (!w && m > 0) {
     ERC_CUDA(cudaMemsetAsync(p.flag, 0, sizeof(int), s));
     k_all_unit<<<grid_for(m, 256), 256, 0, s>>>(p.ew, m, p.flag);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     ERC_CUDA(cudaMemcpyAsync(&nonunit, p.flag, sizeof(int), cudaMemcpyDeviceToHost, s));
     ERC_CUDA(cudaStreamSynchronize(s));
@@ -149,6 +158,7 @@ using namespace erc;
 
 extern "C" const char* erc_version(void) { return "erc-gb300 0.1 (sm_103a)"; }
 extern "C" const char* erc_last_error(void) { return g_err; }
+extern "C" uint64_t erc_kernel_launches(void) { return g_launches.load(); }
 
 extern "C" size_t erc_run_workspace_size(int32_t n, int64_t m_in, int32_t kc) {
   if (n < 1 || m_in < 0 || kc < 1) return 0;

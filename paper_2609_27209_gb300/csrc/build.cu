@@ -214,28 +214,35 @@ extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const i
   const uint64_t sent = (2 * B >= 64) ? ~0ull : ((1ull << (2 * B)) - 1ull);
   if (m_in > 0) {
     k_emit<<<grid_for(m_in, BT), BT, 0, s>>>(src, dst, w, m_in, n, B, sent, p.keys, p.vals, p.err);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     ERC_TRY(radix_sort_pairs(p.keys, p.vals, p.keys_alt, p.vals_alt, E, 2 * B, p.sort_tmp, s));
     k_heads<<<grid_for(E, BT), BT, 0, s>>>(p.keys, E, sent, p.head);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     ERC_TRY(exclusive_scan_i64(nullptr, p.head, p.slot, E, &p.counters[0], p.scan_tmp, s));
     ERC_CUDA(cudaMemsetAsync(p.upper, 0, (size_t)E, s));  // slots past nnz must not count
     k_emit_csr<<<grid_for(E, BT), BT, 0, s>>>(p.keys, p.vals, p.head, p.slot, w, E, B,
                                               dup_policy == ERC_DUP_FIRST, col, p.wmerged,
                                               p.row_of, p.upper);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     k_row_ptr<<<grid_for(E, BT), BT, 0, s>>>(p.row_of, p.counters, n, row_ptr);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
   k_degree<<<grid_for(n, BT), BT, 0, s>>>(row_ptr, p.wmerged, n, deg, val, p.counters);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   if (m_in > 0) {
     ERC_TRY(exclusive_scan_i64(nullptr, p.upper, p.eidx, E, &p.counters[1], p.scan_tmp, s));
     k_emit_edges<<<grid_for(E, BT), BT, 0, s>>>(p.upper, p.eidx, p.row_of, col, p.wmerged,
                                                 p.counters, eu, ev, ew, csr_eid);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     k_lower_eid<<<grid_for(E, BT), BT, 0, s>>>(p.upper, p.row_of, col, row_ptr, p.counters,
                                                csr_eid);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
   int64_t h_counters[2] = {0, 0};

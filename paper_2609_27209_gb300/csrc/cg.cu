@@ -426,6 +426,7 @@ erc_status launch_spmm(const SpmmArgs& a, cudaStream_t s) {
       k_spmm<LPR, VPL, true, MODE><<<grid, T, 0, s>>>(a);
     else
       k_spmm<LPR, VPL, false, MODE><<<grid, T, 0, s>>>(a);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     return ERC_OK;
   });
@@ -437,8 +438,10 @@ erc_status launch_iteration(const SpmmArgs& sa, const VecArgs& va, cudaStream_t 
   ERC_TRY(launch_spmm<MODE_STEP>(sa, s));
   const int nvec = va.ld / 4;
   k_update_xr<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_update_p<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
 }
@@ -501,8 +504,10 @@ erc_status iteration_graph(const SpmmArgs& sa, const VecArgs& va, int S, cudaGra
   cudaStream_t cs = capture_stream();
   if (!cs) return set_error(ERC_ERR_CUDA, "no capture stream");
   ERC_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  set_capturing(true);
   erc_status st = ERC_OK;
   for (int i = 0; i < S && st == ERC_OK; ++i) st = launch_iteration(sa, va, cs);
+  set_capturing(false);
   cudaGraph_t graph = nullptr;
   cudaError_t ce = cudaStreamEndCapture(cs, &graph);
   if (st != ERC_OK) {
@@ -617,6 +622,7 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
 
   const int nvec = ld / 4;
   k_cg_init<<<vec_grid(g->n, nvec), vec_threads(nvec), 0, s>>>(va);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
 
   const int S = iterations_per_poll(g, ld);
@@ -626,6 +632,7 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   int h_any = 1;
   while (done < max_iter) {
     ERC_CUDA(cudaGraphLaunch(exec, s));
+    count_launches(3LL * S);  // the graph holds S iterations of three kernels
     done += S;
     ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
     ERC_CUDA(cudaStreamSynchronize(s));

@@ -288,6 +288,7 @@ extern "C" erc_status erc_edge_resistance(const erc_graph* g, const float* X, in
     const int64_t nseg = (g->m + 31) / 32;
     k_edge_resistance<LPR, VPL><<<grid_for(nseg, T / LPR), T, 0, s>>>(g->eu, g->ev, g->m, X, ld,
                                                                        kc, R_acc);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     return ERC_OK;
   });
@@ -305,9 +306,11 @@ extern "C" erc_status erc_curvature(const erc_graph* g, const float* R, float* p
   else
     k_node_curvature<false><<<grid_for(g->n, T / 32), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
                                                                  R, g->n, p_node);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   if (g->m > 0) {
     k_edge_curvature<<<grid_for(g->m, T), T, 0, s>>>(g->eu, g->ev, p_node, R, g->m, kappa);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
   return ERC_OK;
@@ -341,19 +344,25 @@ extern "C" erc_status erc_sampling_probs(const erc_graph* g, const float* kappa,
   }
   const int ge = grid_for(g->m, T);
   k_kappa_minmax<<<ge, T, 0, s>>>(kappa, g->m, w.part_min, w.part_max);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_minmax_final<<<1, T, 0, s>>>(w.part_min, w.part_max, ge, w.scal);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   const int gn = grid_for(g->n, T / 32);
   k_qnode<<<gn, T, 0, s>>>(g->row_ptr, g->csr_eid, kappa, g->n, (double)eta, w.scal, w.qnode,
                            w.part_qn, w.part_cnt);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_qedge<<<ge, T, 0, s>>>(kappa, g->m, w.scal, w.part_qe);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_sums_final<<<1, T, 0, s>>>(w.part_qn, w.part_cnt, gn, w.part_qe, ge, w.scal);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_normalize<<<grid_for(g->n > g->m ? g->n : g->m, T), T, 0, s>>>(
       g->row_ptr, w.qnode, g->n, kappa, g->m, w.scal, prob_node, prob_edge);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
 }

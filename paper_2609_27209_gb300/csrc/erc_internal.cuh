@@ -42,6 +42,11 @@ inline cudaStream_t as_stream(erc_stream s) { return reinterpret_cast<cudaStream
 // SM count of the current device (cached per device).
 int sm_count();
 
+// process-wide count of kernels this library has launched (graph launches add the kernels they
+// contain); launches recorded while a graph is being captured are not counted
+void count_launches(long long k);
+void set_capturing(bool on);
+
 // ------------------------------------------------------------------------------------------------
 // workspace carving: the same plan runs once to size (base == nullptr) and once to carve
 // ------------------------------------------------------------------------------------------------

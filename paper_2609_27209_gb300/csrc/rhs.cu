@@ -129,6 +129,7 @@ extern "C" erc_status erc_jl_rhs(const erc_graph* g, uint64_t seed, int32_t K, i
     else
       k_jl_rhs<LPR, VPL, false><<<grid, 256, 0, s>>>(g->row_ptr, g->col, g->val, g->csr_eid, g->n,
                                                      key, inv_sqrt_k, c0, kc, ld, Y);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     return ERC_OK;
   });
@@ -144,6 +145,7 @@ extern "C" erc_status erc_philox_signs(uint64_t seed, int64_t e0, int64_t e1, in
   const uint2 key = make_uint2((uint32_t)(seed & 0xffffffffu), (uint32_t)(seed >> 32));
   k_philox_signs<<<grid_for(total, 256), 256, 0, as_stream(stream)>>>(key, e0, e1, c0, c1,
                                                                       out_bits);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
 }

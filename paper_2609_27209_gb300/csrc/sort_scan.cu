@@ -113,15 +113,18 @@ erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* 
   int64_t nb = scan_blocks(n);
   if (nb == 1) {
     k_scan_apply<<<1, SCAN_THREADS, 0, s>>>(in, n, (const int64_t*)nullptr, out, total);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     return ERC_OK;
   }
   int64_t* sums = tmp;
   int64_t* rest = tmp + ((nb + 31) & ~int64_t(31));
   k_scan_reduce<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, sums);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   ERC_TRY(scan_impl(LoadI64{sums}, nb, sums, (int64_t*)nullptr, rest, s));
   k_scan_apply<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, sums, out, total);
+  count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
 }
@@ -246,9 +249,11 @@ erc_status radix_sort_pairs(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, 
   int passes = 0;
   for (int shift = 0; shift < bits; shift += 8, ++passes) {
     k_radix_hist<<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, n, shift, counts, nb);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     ERC_TRY(exclusive_scan_i64(counts, nullptr, offs, (int64_t)cnt, nullptr, scan_tmp, s));
     k_radix_scatter<<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, va, kb, vb, n, shift, offs, nb);
+    count_launches(1);
     ERC_CUDA(cudaGetLastError());
     std::swap(ka, kb);
     std::swap(va, vb);

@@ -53,6 +53,7 @@ class ErcParamsC(ctypes.Structure):
 _SIGS = {
     "erc_version": (ctypes.c_char_p, []),
     "erc_last_error": (ctypes.c_char_p, []),
+    "erc_kernel_launches": (ctypes.c_uint64, []),
     "erc_build_laplacian_workspace_size": (_sz, [_i32, _i64]),
     "erc_build_laplacian": (_i32, [_i32, _c_p, _c_p, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, ctypes.POINTER(_i64), _c_p, _sz, _c_p]),
@@ -122,6 +123,10 @@ def _workspace(nbytes, device):
 
 def erc_version():
     return lib().erc_version().decode()
+
+
+def erc_kernel_launches():
+    return int(lib().erc_kernel_launches())
 
 
 @dataclass
