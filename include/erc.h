@@ -173,6 +173,13 @@ erc_status erc_laplacian_apply(const erc_graph* g, float eps, const float* P, fl
                                int32_t ld, int32_t kc, double* pAp, void* ws, size_t ws_bytes,
                                erc_stream s);
 
+/* erc_laplacian_apply_timed -- benchmarking helper: one untimed erc_laplacian_apply, then `reps`
+ * back-to-back launches of the operator kernel alone between two CUDA events recorded on `s`;
+ * *avg_us (host) receives the mean launch duration in microseconds.  Synchronises s. */
+erc_status erc_laplacian_apply_timed(const erc_graph* g, float eps, const float* P, float* AP,
+                                     int32_t ld, int32_t kc, double* pAp, int32_t reps,
+                                     float* avg_us, void* ws, size_t ws_bytes, erc_stream s);
+
 /* ---------------------------------------------------------------------------------------------
  * erc_philox_signs -- the sign bits of Q[e, c] for e in [e0, e1), c in [c0, c1) (see erc_jl_rhs),
  * written to out_bits (device, row-major (e1-e0) x (c1-c0), one uint32 0/1 per entry).

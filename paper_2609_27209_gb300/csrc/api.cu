@@ -45,6 +45,30 @@ int sm_count() {
   return cache[dev];
 }
 
+int resident_per_sm(const void* kernel, int threads, size_t smem) {
+  struct Entry {
+    const void* k;
+    int threads, dev, blocks;
+    size_t smem;
+  };
+  static std::mutex mu;
+  static Entry cache[256];
+  static int used = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (cache[i].k == kernel && cache[i].threads == threads && cache[i].dev == dev &&
+        cache[i].smem == smem)
+      return cache[i].blocks;
+  int nb = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kernel, threads, smem) != cudaSuccess ||
+      nb < 1)
+    nb = 1;
+  if (used < 256) cache[used++] = Entry{kernel, threads, dev, nb, smem};
+  return nb;
+}
+
 erc_status check_graph(const erc_graph* g) {
   ERC_REQUIRE(g, "graph is null");
   ERC_REQUIRE(g->n >= 1, "graph has n < 1");

@@ -1,15 +1,18 @@
 // cg.cu -- column-wise CG on L_eps X = Y (Eq. 5, §3.1.3, Algorithm 1) and the operator
 // L_eps P = eps P + (D - A) P it iterates on.
 //
-// One CG iteration is three kernels over the row-major n x ld block:
-//   k_spmm<MODE_STEP>  AP = L_eps P (warp-per-row gather of neighbour rows, float4 along the
-//                      columns), per-column p.Ap partials; the last block forms alpha = rr / pAp.
-//   k_update_xr        x += alpha p, r -= alpha Ap, per-column r.r; the last block forms beta,
-//                      counts the iteration and retires converged columns.
-//   k_update_p         p = r + beta p for the columns still active.
-// Reductions are deterministic (fixed order, float-pair accumulation).  A run of S iterations
-// is captured once into a CUDA graph and relaunched; kernels return at once when no column is
-// active, so the host only polls the "any active" flag between graph launches.
+// One CG iteration is two kernels over the row-major n x ld block:
+//   k_spmm<MODE_STEP>  AP = L_eps P: a group of LPR lanes gathers the neighbour rows of one
+//                      light row (float4 along the columns); rows heavier than H are taken by a
+//                      whole block, its groups splitting the row and combining in a fixed order.
+//                      Per-column p.Ap partials; the last block to finish forms alpha = rr / pAp.
+//   k_update_fused     x += alpha p, r -= alpha Ap and r.r; the last block forms beta, counts the
+//                      iteration and retires converged columns, then releases a grid barrier;
+//                      every block then applies p = r + beta p to its rows.  Launched
+//                      cooperatively (all blocks resident), the barrier wait is bounded.
+// Reductions are deterministic: fixed groupings and orders, float-pair accumulation.  S
+// iterations are captured once into a CUDA graph and relaunched; kernels return at once when no
+// column is active, so the host only polls the "any active" flag between graph launches.
 #include <cstring>
 #include <mutex>
 
@@ -20,15 +23,35 @@ namespace {
 
 constexpr int T = 256;
 constexpr int WARPS = T / 32;
+constexpr int SMEM_FLOATS = 8192;  // 32 KB: heavy-row combine buffer, or the reduction buffers
+constexpr unsigned SPIN_LIMIT = 1u << 24;
 enum { MODE_STEP = 0, MODE_APPLY = 1, MODE_RESID = 2 };
+
+struct HeavyRows {
+  uint8_t* flag;    // [n]
+  int64_t* pos;     // [n]
+  int32_t* list;    // [n] rows with more than H neighbours, ascending
+  int64_t* count;   // [1]
+  void* scan_tmp;
+};
+
+void plan_heavy(Arena& a, HeavyRows& h, int32_t n) {
+  h.flag = a.take<uint8_t>(n);
+  h.pos = a.take<int64_t>(n);
+  h.list = a.take<int32_t>(n);
+  h.count = a.take<int64_t>(1);
+  h.scan_tmp = a.take<char>(scan_temp_bytes(n));
+}
 
 struct CgWork {
   float *R, *P, *AP;
   float *alpha, *beta;
   double *rr, *yy;
   int *active, *conv, *iters;
-  int* flags;  // [0] any column active  [1] numeric trouble  [2] unconverged columns
+  int* flags;  // [0] any column active [1] numeric trouble [2] unconverged columns [3] timeout
+  unsigned* gen;  // generation counter of the update kernel's grid barrier
   ColReduce cr;
+  HeavyRows heavy;
 };
 
 void plan_cg(Arena& a, CgWork& w, int32_t n, int32_t ld) {
@@ -44,7 +67,9 @@ void plan_cg(Arena& a, CgWork& w, int32_t n, int32_t ld) {
   w.conv = a.take<int>(ld);
   w.iters = a.take<int>(ld);
   w.flags = a.take<int>(8);
+  w.gen = a.take<unsigned>(8);
   plan_colreduce(a, w.cr, ld);
+  plan_heavy(a, w.heavy, n);
 }
 
 struct SpmmArgs {
@@ -53,6 +78,9 @@ struct SpmmArgs {
   const float* val;
   int32_t n, ld, kc;
   float eps;
+  int32_t H;               // rows with more than H neighbours are split over a block
+  const int32_t* heavy;    // their ids, ascending
+  const int64_t* nheavy;   // their number (device)
   const float* P;  // operand: P (step/apply) or X (residual)
   float* AP;       // output of step/apply
   const float* Y;  // residual mode
@@ -68,6 +96,11 @@ struct SpmmArgs {
   float* relres_out;
   int32_t* iters_out;
 };
+
+__device__ __forceinline__ float4 ld_f4(const float* p) {
+  return __ldg(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
 
 // per-warp then per-block combination of per-thread column partials of a row-group kernel
 template <int LPR, int VPL>
@@ -106,18 +139,120 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
   }
 }
 
-__device__ __forceinline__ float4 ld_f4(const float* p) {
-  return __ldg(reinterpret_cast<const float4*>(p));
+// acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots
+template <int LPR, int VPL, bool WEIGHTED>
+__device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int nvec,
+                                             const float4 (&pu)[VPL], int64_t j0, int64_t j1,
+                                             float4 (&acc)[VPL]) {
+  constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
+  for (int64_t jb = j0; jb < j1; jb += LPR) {
+    const int64_t jj = jb + gl;
+    int32_t cidx = 0;
+    float wv = 1.f;
+    if (jj < j1) {
+      cidx = __ldg(a.col + jj);
+      if (WEIGHTED) wv = __ldg(a.val + jj);
+    }
+    const int cnt = (int)min((int64_t)LPR, j1 - jb);
+    int t = 0;
+    for (; t + U <= cnt; t += U) {
+      int cj[U];
+      float wj[U];
+      float4 pv[U][VPL];
+#pragma unroll
+      for (int k = 0; k < U; ++k) {
+        cj[k] = __shfl_sync(gm, cidx, t + k, LPR);
+        wj[k] = WEIGHTED ? __shfl_sync(gm, wv, t + k, LPR) : 1.f;
+      }
+#pragma unroll
+      for (int k = 0; k < U; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int q = gl + LPR * v;
+          pv[k][v] = q < nvec ? ld_f4(a.P + (size_t)cj[k] * a.ld + 4 * q) : f4_zero();
+        }
+#pragma unroll
+      for (int k = 0; k < U; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          acc[v].x = fmaf(wj[k], pu[v].x - pv[k][v].x, acc[v].x);
+          acc[v].y = fmaf(wj[k], pu[v].y - pv[k][v].y, acc[v].y);
+          acc[v].z = fmaf(wj[k], pu[v].z - pv[k][v].z, acc[v].z);
+          acc[v].w = fmaf(wj[k], pu[v].w - pv[k][v].w, acc[v].w);
+        }
+    }
+    for (; t < cnt; ++t) {
+      const int c1 = __shfl_sync(gm, cidx, t, LPR);
+      const float w1 = WEIGHTED ? __shfl_sync(gm, wv, t, LPR) : 1.f;
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q < nvec) {
+          const float4 p1 = ld_f4(a.P + (size_t)c1 * a.ld + 4 * q);
+          acc[v].x = fmaf(w1, pu[v].x - p1.x, acc[v].x);
+          acc[v].y = fmaf(w1, pu[v].y - p1.y, acc[v].y);
+          acc[v].z = fmaf(w1, pu[v].z - p1.z, acc[v].z);
+          acc[v].w = fmaf(w1, pu[v].w - p1.w, acc[v].w);
+        }
+      }
+    }
+  }
+}
+
+// L_eps p_u = eps p_u + acc: store it (step/apply) or y_u minus it (residual), and add this
+// lane's column contributions to the dot partials (p.Ap, or |y - L x|^2)
+template <int LPR, int VPL, int MODE>
+__device__ __forceinline__ void finish_row(const SpmmArgs& a, int64_t u, int gl, int nvec,
+                                           const float4 (&pu)[VPL], const float4 (&acc)[VPL],
+                                           float2 (&dot)[VPL][4]) {
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int q = gl + LPR * v;
+    if (q >= nvec) continue;
+    float4 o;
+    o.x = fmaf(a.eps, pu[v].x, acc[v].x);
+    o.y = fmaf(a.eps, pu[v].y, acc[v].y);
+    o.z = fmaf(a.eps, pu[v].z, acc[v].z);
+    o.w = fmaf(a.eps, pu[v].w, acc[v].w);
+    if (MODE == MODE_RESID) {
+      const float4 y = ld_f4(a.Y + (size_t)u * a.ld + 4 * q);
+      const int cb = 4 * q;
+      o.x = cb + 0 < a.kc ? y.x - o.x : 0.f;
+      o.y = cb + 1 < a.kc ? y.y - o.y : 0.f;
+      o.z = cb + 2 < a.kc ? y.z - o.z : 0.f;
+      o.w = cb + 3 < a.kc ? y.w - o.w : 0.f;
+      dot[v][0] = df_fma(dot[v][0], o.x, o.x);
+      dot[v][1] = df_fma(dot[v][1], o.y, o.y);
+      dot[v][2] = df_fma(dot[v][2], o.z, o.z);
+      dot[v][3] = df_fma(dot[v][3], o.w, o.w);
+    } else {
+      reinterpret_cast<float4*>(a.AP + (size_t)u * a.ld)[q] = o;
+      dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
+      dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
+      dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
+      dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
+    }
+  }
+}
+
+template <int LPR, int VPL>
+__device__ __forceinline__ void load_row(const SpmmArgs& a, int64_t u, int gl, int nvec,
+                                         float4 (&pu)[VPL], float4 (&acc)[VPL]) {
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int q = gl + LPR * v;
+    pu[v] = q < nvec ? ld_f4(a.P + (size_t)u * a.ld + 4 * q) : f4_zero();
+    acc[v] = f4_zero();
+  }
 }
 
 template <int LPR, int VPL, bool WEIGHTED, int MODE>
-__global__ void __launch_bounds__(T) k_spmm(SpmmArgs a) {
+__global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(SpmmArgs a) {
   if (MODE == MODE_STEP && *(volatile int*)a.flags == 0) return;
-  __shared__ float2 sbuf[MAX_LD];
-  __shared__ float2 scratch[WARPS * 256];
-  constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
+  __shared__ __align__(16) float smem[SMEM_FLOATS];
+  constexpr int GPB = T / LPR;  // groups per block
   const int gl = threadIdx.x & (LPR - 1);
-  const int gpb = T / LPR;
+  const int gi = threadIdx.x / LPR;
   const int nvec = a.ld >> 2;
   const unsigned gm = group_mask<LPR>();
   float2 dot[VPL][4];
@@ -126,100 +261,58 @@ __global__ void __launch_bounds__(T) k_spmm(SpmmArgs a) {
 #pragma unroll
     for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
 
-  for (int64_t u = (int64_t)blockIdx.x * gpb + threadIdx.x / LPR; u < a.n;
-       u += (int64_t)gridDim.x * gpb) {
-    float4 pu[VPL], acc[VPL];
-#pragma unroll
-    for (int v = 0; v < VPL; ++v) {
-      const int q = gl + LPR * v;
-      pu[v] = q < nvec ? ld_f4(a.P + (size_t)u * a.ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
-      acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+  // heavy rows: one block per row, its GPB groups take equal slices of the neighbour list and
+  // group 0 adds the slices in group order
+  const int64_t nheavy = a.nheavy ? *a.nheavy : 0;
+  for (int64_t h = blockIdx.x; h < nheavy; h += gridDim.x) {
+    const int64_t u = a.heavy[h];
     const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
-    for (int64_t jb = j0; jb < j1; jb += LPR) {
-      const int64_t jj = jb + gl;
-      int32_t cidx = 0;
-      float wv = 1.f;
-      if (jj < j1) {
-        cidx = __ldg(a.col + jj);
-        if (WEIGHTED) wv = __ldg(a.val + jj);
-      }
-      const int cnt = (int)min((int64_t)LPR, j1 - jb);
-      int t = 0;
-      for (; t + U <= cnt; t += U) {
-        int cj[U];
-        float wj[U];
-        float4 pv[U][VPL];
-#pragma unroll
-        for (int k = 0; k < U; ++k) {
-          cj[k] = __shfl_sync(gm, cidx, t + k, LPR);
-          wj[k] = WEIGHTED ? __shfl_sync(gm, wv, t + k, LPR) : 1.f;
-        }
-#pragma unroll
-        for (int k = 0; k < U; ++k)
-#pragma unroll
-          for (int v = 0; v < VPL; ++v) {
-            const int q = gl + LPR * v;
-            pv[k][v] = q < nvec ? ld_f4(a.P + (size_t)cj[k] * a.ld + 4 * q)
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
-          }
-#pragma unroll
-        for (int k = 0; k < U; ++k)
-#pragma unroll
-          for (int v = 0; v < VPL; ++v) {
-            acc[v].x = fmaf(wj[k], pu[v].x - pv[k][v].x, acc[v].x);
-            acc[v].y = fmaf(wj[k], pu[v].y - pv[k][v].y, acc[v].y);
-            acc[v].z = fmaf(wj[k], pu[v].z - pv[k][v].z, acc[v].z);
-            acc[v].w = fmaf(wj[k], pu[v].w - pv[k][v].w, acc[v].w);
-          }
-      }
-      for (; t < cnt; ++t) {
-        const int c1 = __shfl_sync(gm, cidx, t, LPR);
-        const float w1 = WEIGHTED ? __shfl_sync(gm, wv, t, LPR) : 1.f;
-#pragma unroll
-        for (int v = 0; v < VPL; ++v) {
-          const int q = gl + LPR * v;
-          if (q < nvec) {
-            const float4 p1 = ld_f4(a.P + (size_t)c1 * a.ld + 4 * q);
-            acc[v].x = fmaf(w1, pu[v].x - p1.x, acc[v].x);
-            acc[v].y = fmaf(w1, pu[v].y - p1.y, acc[v].y);
-            acc[v].z = fmaf(w1, pu[v].z - p1.z, acc[v].z);
-            acc[v].w = fmaf(w1, pu[v].w - p1.w, acc[v].w);
-          }
-        }
-      }
-    }
+    const int64_t per = (j1 - j0 + GPB - 1) / GPB;
+    const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
+    float4 pu[VPL], acc[VPL];
+    load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, nvec, pu, s0, s1, acc);
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
-      if (q >= nvec) continue;
-      float4 o;  // L_eps p = eps p_u + sum_v w_uv (p_u - p_v)
-      o.x = fmaf(a.eps, pu[v].x, acc[v].x);
-      o.y = fmaf(a.eps, pu[v].y, acc[v].y);
-      o.z = fmaf(a.eps, pu[v].z, acc[v].z);
-      o.w = fmaf(a.eps, pu[v].w, acc[v].w);
-      if (MODE == MODE_RESID) {
-        const float4 y = ld_f4(a.Y + (size_t)u * a.ld + 4 * q);
-        const int cb = 4 * q;
-        o.x = cb + 0 < a.kc ? y.x - o.x : 0.f;
-        o.y = cb + 1 < a.kc ? y.y - o.y : 0.f;
-        o.z = cb + 2 < a.kc ? y.z - o.z : 0.f;
-        o.w = cb + 3 < a.kc ? y.w - o.w : 0.f;
-        dot[v][0] = df_fma(dot[v][0], o.x, o.x);
-        dot[v][1] = df_fma(dot[v][1], o.y, o.y);
-        dot[v][2] = df_fma(dot[v][2], o.z, o.z);
-        dot[v][3] = df_fma(dot[v][3], o.w, o.w);
-      } else {
-        reinterpret_cast<float4*>(a.AP + (size_t)u * a.ld)[q] = o;
-        dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
-        dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
-        dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
-        dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
-      }
+      if (q < nvec) reinterpret_cast<float4*>(smem + gi * a.ld)[q] = acc[v];
     }
+    __syncthreads();
+    if (gi == 0) {
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q >= nvec) continue;
+        float4 s = f4_zero();
+        for (int g = 0; g < GPB; ++g) {
+          const float4 c = reinterpret_cast<const float4*>(smem + g * a.ld)[q];
+          s.x += c.x;
+          s.y += c.y;
+          s.z += c.z;
+          s.w += c.w;
+        }
+        acc[v] = s;
+      }
+      finish_row<LPR, VPL, MODE>(a, u, gl, nvec, pu, acc, dot);
+    }
+    __syncthreads();
+  }
+
+  // light rows: one group per row
+  const int64_t ngroups = (int64_t)gridDim.x * GPB;
+  for (int64_t u = (int64_t)blockIdx.x * GPB + gi; u < a.n; u += ngroups) {
+    const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+    if (j1 - j0 > a.H) continue;
+    float4 pu[VPL], acc[VPL];
+    load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, nvec, pu, j0, j1, acc);
+    finish_row<LPR, VPL, MODE>(a, u, gl, nvec, pu, acc, dot);
   }
   if (MODE == MODE_APPLY && a.pap_out == nullptr) return;
 
+  float2* sbuf = reinterpret_cast<float2*>(smem);
+  float2* scratch = reinterpret_cast<float2*>(smem + 2 * MAX_LD);
+  __syncthreads();
   block_partials_rowgroup<LPR, VPL>(dot, sbuf, scratch, a.ld);
   if (!grid_colreduce(a.cr, sbuf, sbuf, a.ld)) return;
   for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
@@ -261,6 +354,7 @@ struct VecArgs {
   float *alpha, *beta;
   double *rr, *yy;
   int *active, *conv, *iters, *flags;
+  unsigned* gen;
   ColReduce cr;
 };
 
@@ -297,7 +391,7 @@ __global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
     if (cb + 3 >= a.kc) y.w = 0.f;
     *reinterpret_cast<float4*>(a.R + i) = y;
     *reinterpret_cast<float4*>(a.P + i) = y;
-    *reinterpret_cast<float4*>(a.X + i) = make_float4(0.f, 0.f, 0.f, 0.f);
+    *reinterpret_cast<float4*>(a.X + i) = f4_zero();
     d[0] = df_fma(d[0], y.x, y.x);
     d[1] = df_fma(d[1], y.y, y.y);
     d[2] = df_fma(d[2], y.z, y.z);
@@ -331,18 +425,31 @@ __global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
   if (threadIdx.x == 0) a.flags[0] = any;
 }
 
-__global__ void __launch_bounds__(T) k_update_xr(VecArgs a) {
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// x += alpha p, r -= alpha Ap, r.r  |grid barrier: beta, convergence|  p = r + beta p
+__global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   if (*(volatile int*)a.flags == 0) return;
   __shared__ float2 red[T * 4];
   __shared__ float2 sbuf[MAX_LD];
+  __shared__ unsigned s_gen;
+  if (threadIdx.x == 0) s_gen = ld_acquire(a.gen);
   const int nvec = a.ld >> 2, rb = blockDim.x / nvec;
   const int q = threadIdx.x % nvec;
+  const int64_t row0 = (int64_t)blockIdx.x * rb + threadIdx.x / nvec;
+  const int64_t rstep = (int64_t)gridDim.x * rb;
   const float4 al = *reinterpret_cast<const float4*>(a.alpha + 4 * q);
   float2 d[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                  make_float2(0.f, 0.f)};
   if (al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f) {
-    for (int64_t row = (int64_t)blockIdx.x * rb + threadIdx.x / nvec; row < a.n;
-         row += (int64_t)gridDim.x * rb) {
+    for (int64_t row = row0; row < a.n; row += rstep) {
       const size_t i = (size_t)row * a.ld + 4 * q;
       float4 x = *reinterpret_cast<const float4*>(a.X + i);
       float4 r = *reinterpret_cast<const float4*>(a.R + i);
@@ -365,44 +472,52 @@ __global__ void __launch_bounds__(T) k_update_xr(VecArgs a) {
     }
   }
   block_partials_quad(d, red, sbuf, a.ld, nvec);
-  if (!grid_colreduce(a.cr, sbuf, sbuf, a.ld)) return;
-  int any = 0;
-  for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
-    float be = 0.f;
-    if (a.active[c]) {
-      const double rn = df_value(sbuf[c]);
-      const int it = a.iters[c] + 1;
-      a.iters[c] = it;
-      if (!isfinite(rn)) {
-        a.active[c] = 0;
-        atomicOr(&a.flags[1], 1);
-      } else {
-        be = (float)(rn / a.rr[c]);
-        a.rr[c] = rn;
-        if (rn <= a.tol2 * a.yy[c]) {
-          a.conv[c] = 1;
+  if (grid_colreduce(a.cr, sbuf, sbuf, a.ld)) {
+    int any = 0;
+    for (int c = threadIdx.x; c < a.ld; c += blockDim.x) {
+      float be = 0.f;
+      if (a.active[c]) {
+        const double rn = df_value(sbuf[c]);
+        const int it = a.iters[c] + 1;
+        a.iters[c] = it;
+        if (!isfinite(rn)) {
           a.active[c] = 0;
-        } else if (it >= a.max_iter) {
-          a.active[c] = 0;
+          atomicOr(&a.flags[1], 1);
+        } else {
+          be = (float)(rn / a.rr[c]);
+          a.rr[c] = rn;
+          if (rn <= a.tol2 * a.yy[c]) {
+            a.conv[c] = 1;
+            a.active[c] = 0;
+          } else if (it >= a.max_iter) {
+            a.active[c] = 0;
+          }
         }
       }
+      a.beta[c] = be;
+      any |= a.active[c];
     }
-    a.beta[c] = be;
-    any |= a.active[c];
+    any = __syncthreads_or(any);
+    if (threadIdx.x == 0) {
+      a.flags[0] = any;
+      __threadfence();
+      red_release_add(a.gen, 1u);  // release the blocks waiting for beta
+    }
+  } else if (threadIdx.x == 0) {
+    unsigned spins = 0;
+    while (ld_acquire(a.gen) == s_gen) {
+      if (++spins > SPIN_LIMIT) {  // bounded: flag the timeout and fall through
+        atomicOr(&a.flags[3], 1);
+        break;
+      }
+      __nanosleep(64);
+    }
   }
-  any = __syncthreads_or(any);
-  if (threadIdx.x == 0) a.flags[0] = any;
-}
-
-__global__ void __launch_bounds__(T) k_update_p(VecArgs a) {
-  if (*(volatile int*)a.flags == 0) return;
-  const int nvec = a.ld >> 2, rb = blockDim.x / nvec;
-  const int q = threadIdx.x % nvec;
-  const int4 act = *reinterpret_cast<const int4*>(a.active + 4 * q);
+  __syncthreads();
+  const int4 act = __ldcg(reinterpret_cast<const int4*>(a.active + 4 * q));
   if (!(act.x | act.y | act.z | act.w)) return;
-  const float4 be = *reinterpret_cast<const float4*>(a.beta + 4 * q);
-  for (int64_t row = (int64_t)blockIdx.x * rb + threadIdx.x / nvec; row < a.n;
-       row += (int64_t)gridDim.x * rb) {
+  const float4 be = __ldcg(reinterpret_cast<const float4*>(a.beta + 4 * q));
+  for (int64_t row = row0; row < a.n; row += rstep) {
     const size_t i = (size_t)row * a.ld + 4 * q;
     const float4 r = *reinterpret_cast<const float4*>(a.R + i);
     float4 p = *reinterpret_cast<const float4*>(a.P + i);
@@ -414,14 +529,66 @@ __global__ void __launch_bounds__(T) k_update_p(VecArgs a) {
   }
 }
 
+// ---------------------------------------------------------------------------- heavy rows
+__global__ void k_mark_heavy(const int64_t* __restrict__ row_ptr, int32_t n, int32_t H,
+                             uint8_t* __restrict__ flag) {
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n;
+       u += (int64_t)gridDim.x * blockDim.x)
+    flag[u] = (row_ptr[u + 1] - row_ptr[u]) > H;
+}
+__global__ void k_list_heavy(const uint8_t* __restrict__ flag, const int64_t* __restrict__ pos,
+                             int32_t n, int32_t* __restrict__ list) {
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n;
+       u += (int64_t)gridDim.x * blockDim.x)
+    if (flag[u]) list[pos[u]] = (int32_t)u;
+}
+
 // ---------------------------------------------------------------------------- launch helpers
 inline int vec_threads(int nvec) { return nvec * (T / nvec); }
 
 template <int MODE>
-erc_status launch_spmm(const SpmmArgs& a, cudaStream_t s) {
+const void* spmm_kernel(int nvec, bool weighted) {
+  const void* k = nullptr;
+  dispatch_shape(nvec, [&](auto lpr, auto vpl) -> erc_status {
+    constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
+    k = weighted ? (const void*)k_spmm<LPR, VPL, true, MODE>
+                 : (const void*)k_spmm<LPR, VPL, false, MODE>;
+    return ERC_OK;
+  });
+  return k;
+}
+
+// grid and heavy threshold of the operator for this graph: one wave of blocks, and rows heavier
+// than about twice the mean work of a group are split over a block
+void spmm_shape(const erc_graph* g, int ld, int* grid, int32_t* H) {
+  const int nvec = ld / 4;
+  int lpr = nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32;
+  const int gpb = T / lpr;
+  *grid = one_wave_grid(spmm_kernel<MODE_STEP>(nvec, g->val != nullptr), T,
+                        ((long long)g->n + gpb - 1) / gpb);
+  const long long groups = (long long)(*grid) * gpb;
+  long long h = 2 * g->m / (2 * groups);
+  if (h < 32) h = 32;
+  if (h > (1 << 20)) h = 1 << 20;
+  *H = (int32_t)h;
+}
+
+erc_status build_heavy(const erc_graph* g, int32_t H, const HeavyRows& hv, cudaStream_t s) {
+  const int grid = grid_for(g->n, 256);
+  k_mark_heavy<<<grid, 256, 0, s>>>(g->row_ptr, g->n, H, hv.flag);
+  count_launches(1);
+  ERC_CUDA(cudaGetLastError());
+  ERC_TRY(exclusive_scan_i64(nullptr, hv.flag, hv.pos, g->n, hv.count, hv.scan_tmp, s));
+  k_list_heavy<<<grid, 256, 0, s>>>(hv.flag, hv.pos, g->n, hv.list);
+  count_launches(1);
+  ERC_CUDA(cudaGetLastError());
+  return ERC_OK;
+}
+
+template <int MODE>
+erc_status launch_spmm(const SpmmArgs& a, int grid, cudaStream_t s) {
   return dispatch_shape(a.ld / 4, [&](auto lpr, auto vpl) -> erc_status {
     constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
-    const int grid = grid_for(a.n, T / LPR);
     if (a.val)
       k_spmm<LPR, VPL, true, MODE><<<grid, T, 0, s>>>(a);
     else
@@ -432,28 +599,42 @@ erc_status launch_spmm(const SpmmArgs& a, cudaStream_t s) {
   });
 }
 
-inline int vec_grid(int32_t n, int nvec) { return grid_for(n, vec_threads(nvec) / nvec); }
+int update_grid(int32_t n, int nvec) {
+  const int threads = vec_threads(nvec);
+  return one_wave_grid((const void*)k_update_fused, threads,
+                       ((long long)n + threads / nvec - 1) / (threads / nvec));
+}
 
-erc_status launch_iteration(const SpmmArgs& sa, const VecArgs& va, cudaStream_t s) {
-  ERC_TRY(launch_spmm<MODE_STEP>(sa, s));
-  const int nvec = va.ld / 4;
-  k_update_xr<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
+erc_status launch_update(const VecArgs& va, int grid, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(vec_threads(va.ld / 4));
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: the barrier can complete
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ERC_CUDA(cudaLaunchKernelEx(&cfg, k_update_fused, va));
   count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-  k_update_p<<<vec_grid(va.n, nvec), vec_threads(nvec), 0, s>>>(va);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
   return ERC_OK;
+}
+
+erc_status launch_iteration(const SpmmArgs& sa, int sgrid, const VecArgs& va, int ugrid,
+                            cudaStream_t s) {
+  ERC_TRY(launch_spmm<MODE_STEP>(sa, sgrid, s));
+  return launch_update(va, ugrid, s);
 }
 
 // ---------------------------------------------------------------------------- graph cache
 struct GraphKey {
-  const void* ptr[12];
-  long long num[8];
+  const void* ptr[14];
+  long long num[10];
   bool operator==(const GraphKey& o) const {
-    for (int i = 0; i < 12; ++i)
+    for (int i = 0; i < 14; ++i)
       if (ptr[i] != o.ptr[i]) return false;
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < 10; ++i)
       if (num[i] != o.num[i]) return false;
     return true;
   }
@@ -477,19 +658,21 @@ cudaStream_t capture_stream() {
   return cs[dev];
 }
 
-erc_status iteration_graph(const SpmmArgs& sa, const VecArgs& va, int S, cudaGraphExec_t* out) {
+erc_status iteration_graph(const SpmmArgs& sa, int sgrid, const VecArgs& va, int ugrid, int S,
+                           cudaGraphExec_t* out) {
   int dev = 0;
   ERC_CUDA(cudaGetDevice(&dev));
   GraphKey k{};
-  const void* ptrs[12] = {sa.row_ptr, sa.col, sa.val, sa.P, sa.AP, va.X, va.R, va.alpha,
-                          va.active, va.flags, sa.cr.part1, va.Y};
-  for (int i = 0; i < 12; ++i) k.ptr[i] = ptrs[i];
+  const void* ptrs[14] = {sa.row_ptr, sa.col, sa.val, sa.P, sa.AP, va.X, va.R, va.alpha,
+                          va.active, va.flags, sa.cr.part1, va.Y, sa.heavy, va.gen};
+  for (int i = 0; i < 14; ++i) k.ptr[i] = ptrs[i];
   int eps_bits = 0;
   long long tol_bits = 0;
   memcpy(&eps_bits, &sa.eps, sizeof eps_bits);
   memcpy(&tol_bits, &va.tol2, sizeof tol_bits);
-  long long nums[8] = {sa.n, sa.ld, sa.kc, eps_bits, tol_bits, va.max_iter, S, dev};
-  for (int i = 0; i < 8; ++i) k.num[i] = nums[i];
+  long long nums[10] = {sa.n, sa.ld, sa.kc, eps_bits, tol_bits, va.max_iter, S, dev, sgrid,
+                        (long long)ugrid << 32 | (unsigned)sa.H};
+  for (int i = 0; i < 10; ++i) k.num[i] = nums[i];
   std::lock_guard<std::mutex> lock(g_mu);
   ++g_clock;
   int victim = 0;
@@ -506,7 +689,7 @@ erc_status iteration_graph(const SpmmArgs& sa, const VecArgs& va, int S, cudaGra
   ERC_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
   set_capturing(true);
   erc_status st = ERC_OK;
-  for (int i = 0; i < S && st == ERC_OK; ++i) st = launch_iteration(sa, va, cs);
+  for (int i = 0; i < S && st == ERC_OK; ++i) st = launch_iteration(sa, sgrid, va, ugrid, cs);
   set_capturing(false);
   cudaGraph_t graph = nullptr;
   cudaError_t ce = cudaStreamEndCapture(cs, &graph);
@@ -530,15 +713,13 @@ erc_status iteration_graph(const SpmmArgs& sa, const VecArgs& va, int S, cudaGra
 
 int iterations_per_poll(const erc_graph* g, int ld) {
   const double bytes = (double)(2 * g->m + g->n) * ld * 4.0;  // gathered + streamed per iteration
-  if (bytes < 64e6) return 32;
-  if (bytes < 1e9) return 8;
+  if (bytes < 256e6) return 16;
+  if (bytes < 2e9) return 4;
   return 2;
 }
 
-erc_status check_block(const erc_graph* g, const float* p, int ld, const char* name) {
+erc_status check_block(const float* p, const char* name) {
   ERC_REQUIRE(p && (reinterpret_cast<uintptr_t>(p) & 15) == 0, "%s must be 16-byte aligned", name);
-  (void)g;
-  (void)ld;
   return ERC_OK;
 }
 
@@ -566,8 +747,8 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   ERC_REQUIRE(tol >= 0.f && isfinite(tol), "tol must be finite and >= 0");
   ERC_REQUIRE(max_iter >= 1, "max_iter must be >= 1");
   ERC_REQUIRE(iters && relres, "iters and relres are required");
-  ERC_TRY(check_block(g, Y, ld, "Y"));
-  ERC_TRY(check_block(g, X, ld, "X"));
+  ERC_TRY(check_block(Y, "Y"));
+  ERC_TRY(check_block(X, "X"));
   if (ws_bytes < erc_batched_cg_workspace_size(g->n, ld))
     return set_error(ERC_ERR_CAPACITY, "workspace too small");
   cudaStream_t s = as_stream(stream);
@@ -576,6 +757,14 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   plan_cg(ar, w, g->n, ld);
   ERC_CUDA(cudaMemsetAsync(w.cr.cnt, 0, colreduce_counter_bytes(), s));
   ERC_CUDA(cudaMemsetAsync(w.flags, 0, 8 * sizeof(int), s));
+  ERC_CUDA(cudaMemsetAsync(w.gen, 0, 8 * sizeof(unsigned), s));
+
+  int sgrid = 1;
+  int32_t H = 0;
+  spmm_shape(g, ld, &sgrid, &H);
+  ERC_TRY(build_heavy(g, H, w.heavy, s));
+  const int nvec = ld / 4;
+  const int ugrid = update_grid(g->n, nvec);
 
   VecArgs va{};
   va.n = g->n;
@@ -596,6 +785,7 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   va.conv = w.conv;
   va.iters = w.iters;
   va.flags = w.flags;
+  va.gen = w.gen;
   va.cr = w.cr;
 
   SpmmArgs sa{};
@@ -606,6 +796,9 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   sa.ld = ld;
   sa.kc = kc;
   sa.eps = eps;
+  sa.H = H;
+  sa.heavy = w.heavy.list;
+  sa.nheavy = w.heavy.count;
   sa.P = w.P;
   sa.AP = w.AP;
   sa.Y = Y;
@@ -620,19 +813,18 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   sa.relres_out = relres;
   sa.iters_out = iters;
 
-  const int nvec = ld / 4;
-  k_cg_init<<<vec_grid(g->n, nvec), vec_threads(nvec), 0, s>>>(va);
+  k_cg_init<<<grid_for(g->n, vec_threads(nvec) / nvec), vec_threads(nvec), 0, s>>>(va);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
 
   const int S = iterations_per_poll(g, ld);
   cudaGraphExec_t exec = nullptr;
-  ERC_TRY(iteration_graph(sa, va, S, &exec));
+  ERC_TRY(iteration_graph(sa, sgrid, va, ugrid, S, &exec));
   int done = 0;
   int h_any = 1;
   while (done < max_iter) {
     ERC_CUDA(cudaGraphLaunch(exec, s));
-    count_launches(3LL * S);  // the graph holds S iterations of three kernels
+    count_launches(2LL * S);  // the graph holds S iterations of two kernels
     done += S;
     ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
     ERC_CUDA(cudaStreamSynchronize(s));
@@ -642,10 +834,11 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   // true residual of the returned iterate, plus the per-column outputs
   SpmmArgs ra = sa;
   ra.P = X;
-  ERC_TRY(launch_spmm<MODE_RESID>(ra, s));
-  int h_flags[3] = {0, 0, 0};
-  ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 3 * sizeof(int), cudaMemcpyDeviceToHost, s));
+  ERC_TRY(launch_spmm<MODE_RESID>(ra, sgrid, s));
+  int h_flags[4] = {0, 0, 0, 0};
+  ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 4 * sizeof(int), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
+  if (h_flags[3]) return set_error(ERC_ERR_TIMEOUT, "update kernel grid barrier timed out");
   if (h_flags[1]) return set_error(ERC_ERR_NUMERIC, "non-finite or non-positive CG scalar");
   if (h_flags[2])
     return set_error(ERC_ERR_NOT_CONVERGED, "%d of %d columns reached max_iter=%d", h_flags[2],
@@ -654,11 +847,12 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
 }
 
 extern "C" size_t erc_laplacian_apply_workspace_size(int32_t n, int32_t ld) {
-  (void)n;
-  if (ld < 4) return 0;
+  if (n < 1 || ld < 4) return 0;
   Arena a(nullptr);
   ColReduce cr;
   plan_colreduce(a, cr, ld);
+  HeavyRows h;
+  plan_heavy(a, h, n);
   return a.used + 256;
 }
 
@@ -669,10 +863,16 @@ extern "C" erc_status erc_laplacian_apply(const erc_graph* g, float eps, const f
   ERC_TRY(check_graph(g));
   ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
   ERC_REQUIRE(eps >= 0.f && isfinite(eps), "eps must be finite and >= 0");
-  ERC_TRY(check_block(g, P, ld, "P"));
-  ERC_TRY(check_block(g, AP, ld, "AP"));
+  ERC_TRY(check_block(P, "P"));
+  ERC_TRY(check_block(AP, "AP"));
+  if (ws_bytes < erc_laplacian_apply_workspace_size(g->n, ld))
+    return set_error(ERC_ERR_CAPACITY, "workspace too small");
   cudaStream_t s = as_stream(stream);
+  Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
   SpmmArgs sa{};
+  plan_colreduce(ar, sa.cr, ld);
+  HeavyRows hv;
+  plan_heavy(ar, hv, g->n);
   sa.row_ptr = g->row_ptr;
   sa.col = g->col;
   sa.val = g->val;
@@ -683,12 +883,58 @@ extern "C" erc_status erc_laplacian_apply(const erc_graph* g, float eps, const f
   sa.P = P;
   sa.AP = AP;
   sa.pap_out = pAp;
-  if (pAp) {
-    if (ws_bytes < erc_laplacian_apply_workspace_size(g->n, ld))
-      return set_error(ERC_ERR_CAPACITY, "workspace too small");
-    Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
-    plan_colreduce(ar, sa.cr, ld);
-    ERC_CUDA(cudaMemsetAsync(sa.cr.cnt, 0, colreduce_counter_bytes(), s));
-  }
-  return launch_spmm<MODE_APPLY>(sa, s);
+  int sgrid = 1;
+  spmm_shape(g, ld, &sgrid, &sa.H);
+  sa.heavy = hv.list;
+  sa.nheavy = hv.count;
+  ERC_TRY(build_heavy(g, sa.H, hv, s));
+  if (pAp) ERC_CUDA(cudaMemsetAsync(sa.cr.cnt, 0, colreduce_counter_bytes(), s));
+  return launch_spmm<MODE_APPLY>(sa, sgrid, s);
+}
+
+extern "C" erc_status erc_laplacian_apply_timed(const erc_graph* g, float eps, const float* P,
+                                                float* AP, int32_t ld, int32_t kc, double* pAp,
+                                                int32_t reps, float* avg_us, void* ws,
+                                                size_t ws_bytes, erc_stream stream) {
+  clear_error();
+  ERC_REQUIRE(reps >= 1 && avg_us, "reps >= 1 and avg_us are required");
+  // one untimed call builds the heavy-row list in the workspace and warms the caches
+  ERC_TRY(erc_laplacian_apply(g, eps, P, AP, ld, kc, pAp, ws, ws_bytes, stream));
+  cudaStream_t s = as_stream(stream);
+  Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  SpmmArgs sa{};
+  plan_colreduce(ar, sa.cr, ld);
+  HeavyRows hv;
+  plan_heavy(ar, hv, g->n);
+  sa.row_ptr = g->row_ptr;
+  sa.col = g->col;
+  sa.val = g->val;
+  sa.n = g->n;
+  sa.ld = ld;
+  sa.kc = kc;
+  sa.eps = eps;
+  sa.P = P;
+  sa.AP = AP;
+  sa.pap_out = pAp;
+  int sgrid = 1;
+  spmm_shape(g, ld, &sgrid, &sa.H);
+  sa.heavy = hv.list;
+  sa.nheavy = hv.count;
+  cudaEvent_t e0, e1;
+  ERC_CUDA(cudaEventCreate(&e0));
+  ERC_CUDA(cudaEventCreate(&e1));
+  erc_status st = ERC_OK;
+  cudaError_t ce = cudaEventRecord(e0, s);
+  for (int r = 0; r < reps && st == ERC_OK && ce == cudaSuccess; ++r)
+    st = launch_spmm<MODE_APPLY>(sa, sgrid, s);
+  if (ce == cudaSuccess) ce = cudaEventRecord(e1, s);
+  if (ce == cudaSuccess) ce = cudaEventSynchronize(e1);
+  float ms = 0.f;
+  if (ce == cudaSuccess) ce = cudaEventElapsedTime(&ms, e0, e1);
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  if (st != ERC_OK) return st;
+  if (ce != cudaSuccess) return set_error(ERC_ERR_CUDA, "event timing: %s", cudaGetErrorString(ce));
+  *avg_us = 1000.f * ms / (float)reps;
+  return ERC_OK;
 }

@@ -134,7 +134,12 @@ __device__ __forceinline__ bool grid_colreduce(const ColReduce& cr, const float2
   for (int c = threadIdx.x; c < ld; c += blockDim.x) {
     float2 acc = make_float2(0.f, 0.f);
     const float2* src = cr.part1 + (size_t)grp * RED_GROUP * ld + c;
-    for (int k = 0; k < gsize; ++k) acc = df_add(acc, __ldcg(src + (size_t)k * ld));
+    float2 v[RED_GROUP];  // issue every load before the (ordered) additions
+#pragma unroll
+    for (int k = 0; k < RED_GROUP; ++k)
+      v[k] = k < gsize ? __ldcg(src + (size_t)k * ld) : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < RED_GROUP; ++k) acc = df_add(acc, v[k]);
     cr.part2[(size_t)grp * ld + c] = acc;
   }
   __threadfence();
@@ -148,7 +153,14 @@ __device__ __forceinline__ bool grid_colreduce(const ColReduce& cr, const float2
   __threadfence();
   for (int c = threadIdx.x; c < ld; c += blockDim.x) {
     float2 acc = make_float2(0.f, 0.f);
-    for (int k = 0; k < ng; ++k) acc = df_add(acc, __ldcg(cr.part2 + (size_t)k * ld + c));
+    for (int k0 = 0; k0 < ng; k0 += 16) {
+      float2 v[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k)
+        v[k] = k0 + k < ng ? __ldcg(cr.part2 + (size_t)(k0 + k) * ld + c) : make_float2(0.f, 0.f);
+#pragma unroll
+      for (int k = 0; k < 16; ++k) acc = df_add(acc, v[k]);
+    }
     res[c] = acc;
   }
   if (threadIdx.x == 0) cr.cnt[ng] = 0;
@@ -185,6 +197,17 @@ __device__ __forceinline__ unsigned group_mask() {
     const unsigned lane = threadIdx.x & 31u;
     return ((1u << LPR) - 1u) << (lane & ~(unsigned)(LPR - 1));
   }
+}
+
+// blocks of `kernel` that fit on one SM at `threads` threads (cached per kernel and device)
+int resident_per_sm(const void* kernel, int threads, size_t smem = 0);
+
+// a one-wave grid: min(resident blocks on the whole GPU, blocks the work needs), at least 1
+inline int one_wave_grid(const void* kernel, int threads, long long work_blocks) {
+  long long g = (long long)resident_per_sm(kernel, threads) * sm_count();
+  if (work_blocks < g) g = work_blocks;
+  if (g > MAX_GRID) g = MAX_GRID;
+  return g < 1 ? 1 : (int)g;
 }
 
 // grid size for a grid-stride kernel: at most `waves` resident waves of blocks, at least 1

@@ -69,6 +69,9 @@ _SIGS = {
     "erc_laplacian_apply_workspace_size": (_sz, [_i32, _i32]),
     "erc_laplacian_apply": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _c_p,
                                    _c_p, _sz, _c_p]),
+    "erc_laplacian_apply_timed": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32,
+                                         _i32, _c_p, _i32, ctypes.POINTER(_f32), _c_p, _sz,
+                                         _c_p]),
     "erc_philox_signs": (_i32, [_u64, _i64, _i64, _i32, _i32, _c_p, _c_p]),
     "erc_run_workspace_size": (_sz, [_i32, _i64, _i32]),
     "erc_run": (_i32, [ctypes.POINTER(ErcParamsC), _i32, _c_p, _c_p, _c_p, _i64,
@@ -245,6 +248,20 @@ def erc_laplacian_apply(g, eps, P, kc, want_pap=False):
     _check(lib().erc_laplacian_apply(ctypes.byref(gc), eps, _ptr(P), _ptr(AP), ld, kc, _ptr(pap),
                                      _ptr(ws), ws.numel(), _stream()))
     return AP, pap
+
+
+def erc_laplacian_apply_timed(g, eps, P, kc, reps=50):
+    """Mean duration (microseconds) of the operator kernel over `reps` back-to-back launches."""
+    n, ld = P.shape
+    AP = torch.empty_like(P)
+    pap = torch.empty(kc, dtype=torch.float64, device=P.device)
+    ws = _workspace(lib().erc_laplacian_apply_workspace_size(n, ld), P.device)
+    us = _f32(0)
+    gc = g.c()
+    _check(lib().erc_laplacian_apply_timed(ctypes.byref(gc), eps, _ptr(P), _ptr(AP), ld, kc,
+                                           _ptr(pap), reps, ctypes.byref(us), _ptr(ws),
+                                           ws.numel(), _stream()))
+    return float(us.value)
 
 
 def erc_philox_signs(seed, e0, e1, c0, c1, device="cuda"):
