@@ -13,6 +13,7 @@
 // Reductions are deterministic: fixed groupings and orders, float-pair accumulation.  S
 // iterations are captured once into a CUDA graph and relaunched; kernels return at once when no
 // column is active, so the host only polls the "any active" flag between graph launches.
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -102,6 +103,44 @@ __device__ __forceinline__ float4 ld_f4(const float* p) {
 }
 __device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
 
+// per-warp then per-block combination of per-thread column partials of a row-group kernel with
+// NW warps; the cross-warp step runs over chunks of CH columns (scratch holds NW x CH)
+template <int LPR, int VPL, int NW, int CH>
+__device__ __forceinline__ void block_partials_groups(float2 (&d)[VPL][4], float2* sbuf,
+                                                      float2* scratch, int ld) {
+#pragma unroll
+  for (int off = LPR; off < 32; off <<= 1) {
+#pragma unroll
+    for (int v = 0; v < VPL; ++v)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        float2 o;
+        o.x = __shfl_xor_sync(0xffffffffu, d[v][t].x, off);
+        o.y = __shfl_xor_sync(0xffffffffu, d[v][t].y, off);
+        d[v][t] = df_add(d[v][t], o);
+      }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int cb = 0; cb < ld; cb += CH) {
+    if (lane < LPR) {
+#pragma unroll
+      for (int v = 0; v < VPL; ++v)
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int c = 4 * (lane + LPR * v) + t;
+          if (c >= cb && c < cb + CH && c < ld) scratch[warp * CH + (c - cb)] = d[v][t];
+        }
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < CH && cb + c < ld; c += blockDim.x) {
+      float2 acc = make_float2(0.f, 0.f);
+      for (int w = 0; w < NW; ++w) acc = df_add(acc, scratch[w * CH + c]);
+      sbuf[cb + c] = acc;
+    }
+    __syncthreads();
+  }
+}
+
 // per-warp then per-block combination of per-thread column partials of a row-group kernel
 template <int LPR, int VPL>
 __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], float2* sbuf,
@@ -139,8 +178,9 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
   }
 }
 
-// acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots
-template <int LPR, int VPL, bool WEIGHTED>
+// acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots.
+// L2ONLY loads p through L2 only: required where p is rewritten within the same launch.
+template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false>
 __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int nvec,
                                              const float4 (&pu)[VPL], int64_t j0, int64_t j1,
                                              float4 (&acc)[VPL]) {
@@ -154,22 +194,27 @@ __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned
       if (WEIGHTED) wv = __ldg(a.val + jj);
     }
     const int cnt = (int)min((int64_t)LPR, j1 - jb);
-    int t = 0;
-    for (; t + U <= cnt; t += U) {
+    // batches of U neighbour rows, the last one predicated: every load of a batch is issued
+    // before the first FMA, so a row costs ceil(deg / U) dependent trips
+    for (int t = 0; t < cnt; t += U) {
       int cj[U];
       float wj[U];
       float4 pv[U][VPL];
 #pragma unroll
       for (int k = 0; k < U; ++k) {
-        cj[k] = __shfl_sync(gm, cidx, t + k, LPR);
-        wj[k] = WEIGHTED ? __shfl_sync(gm, wv, t + k, LPR) : 1.f;
+        cj[k] = __shfl_sync(gm, cidx, (t + k) & (LPR - 1), LPR);
+        wj[k] = WEIGHTED ? __shfl_sync(gm, wv, (t + k) & (LPR - 1), LPR) : 1.f;
+        if (t + k >= cnt) wj[k] = 0.f;
       }
 #pragma unroll
       for (int k = 0; k < U; ++k)
 #pragma unroll
         for (int v = 0; v < VPL; ++v) {
           const int q = gl + LPR * v;
-          pv[k][v] = q < nvec ? ld_f4(a.P + (size_t)cj[k] * a.ld + 4 * q) : f4_zero();
+          const float* src = a.P + (size_t)cj[k] * a.ld + 4 * q;
+          pv[k][v] = (q < nvec && t + k < cnt)
+                         ? (L2ONLY ? __ldcg(reinterpret_cast<const float4*>(src)) : ld_f4(src))
+                         : pu[v];
         }
 #pragma unroll
       for (int k = 0; k < U; ++k)
@@ -180,21 +225,6 @@ __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned
           acc[v].z = fmaf(wj[k], pu[v].z - pv[k][v].z, acc[v].z);
           acc[v].w = fmaf(wj[k], pu[v].w - pv[k][v].w, acc[v].w);
         }
-    }
-    for (; t < cnt; ++t) {
-      const int c1 = __shfl_sync(gm, cidx, t, LPR);
-      const float w1 = WEIGHTED ? __shfl_sync(gm, wv, t, LPR) : 1.f;
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        if (q < nvec) {
-          const float4 p1 = ld_f4(a.P + (size_t)c1 * a.ld + 4 * q);
-          acc[v].x = fmaf(w1, pu[v].x - p1.x, acc[v].x);
-          acc[v].y = fmaf(w1, pu[v].y - p1.y, acc[v].y);
-          acc[v].z = fmaf(w1, pu[v].z - p1.z, acc[v].z);
-          acc[v].w = fmaf(w1, pu[v].w - p1.w, acc[v].w);
-        }
-      }
     }
   }
 }
@@ -529,6 +559,313 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   }
 }
 
+// ---------------------------------------------------------------------------- resident CG
+// When r and Ap of every row fit in the SMs' shared memory, one cooperative launch runs the whole
+// solve.  Block b owns rows [b rb, b rb + rb): their r and Ap live in its shared memory, x and p
+// in global memory (p is gathered by other blocks).  Per iteration:
+//   A  Ap = L_eps p for own rows (heavy rows by the whole block), p.Ap   -> reduce, alpha
+//   B  x += alpha p, r -= alpha Ap, r.r                                  -> reduce, beta, stop test
+//   C  p = r + beta p                                                    -> barrier
+// Every reduce and barrier is a bounded wait on one generation counter.  Data written by other
+// blocks inside the launch (p, scalars) is read through L2 (ld.global.cg), never through L1.
+constexpr int PT = 512;
+constexpr int PWARPS = PT / 32;
+constexpr int PCH = 64;
+
+struct ResArgs {
+  SpmmArgs s;
+  VecArgs v;
+  int32_t rb;  // rows per block
+};
+
+__device__ __forceinline__ float4 ldcg_f4(const float* p) {
+  return __ldcg(reinterpret_cast<const float4*>(p));
+}
+
+// wait until the generation counter moves past `g` (bounded; sets flags[3] on timeout)
+__device__ __forceinline__ void wait_generation(unsigned* gen, unsigned g, int* flags) {
+  if (threadIdx.x == 0) {
+    unsigned spins = 0;
+    while (ld_acquire(gen) == g) {
+      if (++spins > SPIN_LIMIT) {
+        atomicOr(&flags[3], 1);
+        break;
+      }
+      __nanosleep(32);
+    }
+  }
+  __syncthreads();
+}
+
+// plain grid barrier on (count, generation); every block calls it the same number of times
+__device__ __forceinline__ void grid_barrier(unsigned* cnt, unsigned* gen, int* flags) {
+  __shared__ unsigned s_g;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    s_g = ld_acquire(gen);
+    __threadfence();
+    if (atomicAdd(cnt, 1u) == gridDim.x - 1) {
+      atomicExch(cnt, 0u);
+      red_release_add(gen, 1u);
+    }
+  }
+  __syncthreads();
+  wait_generation(gen, s_g, flags);
+}
+
+template <int LPR, int VPL, bool WEIGHTED>
+__global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
+  extern __shared__ __align__(16) float dsm[];
+  const SpmmArgs& a = ra.s;
+  const VecArgs& va = ra.v;
+  constexpr int GPB = PT / LPR;
+  const int gl = threadIdx.x & (LPR - 1);
+  const int gi = threadIdx.x / LPR;
+  const int ld = a.ld, nvec = ld >> 2;
+  const unsigned gm = group_mask<LPR>();
+  const int64_t r0 = (int64_t)blockIdx.x * ra.rb;
+  const int nrows = (int)max((int64_t)0, min((int64_t)a.n, r0 + ra.rb) - r0);
+  float* rs = dsm;                                     // [rb][ld]  r of own rows
+  float* aps = rs + (size_t)ra.rb * ld;                // [rb][ld]  Ap of own rows
+  float* comb = aps + (size_t)ra.rb * ld;              // [GPB][ld] heavy-row slices
+  float2* sbuf = reinterpret_cast<float2*>(comb + (size_t)GPB * ld);  // [ld]
+  float2* scratch = sbuf + ld;                         // [PWARPS][PCH]
+  __shared__ unsigned s_gen;
+  __shared__ int64_t s_h0, s_h1;
+  unsigned* bar_cnt = va.gen + 1;
+
+  for (int idx = threadIdx.x; idx < nrows * nvec; idx += PT) {
+    const int i = idx / nvec, q = idx % nvec;
+    reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = ldcg_f4(va.R + (size_t)(r0 + i) * ld + 4 * q);
+  }
+  if (threadIdx.x == 0) {  // this block's slice of the ascending heavy-row list
+    const int64_t nh = a.nheavy ? *a.nheavy : 0;
+    int64_t lo = 0, hi = nh;
+    while (lo < hi) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (a.heavy[mid] < r0) lo = mid + 1; else hi = mid;
+    }
+    s_h0 = lo;
+    hi = nh;
+    while (lo < hi) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (a.heavy[mid] < r0 + nrows) lo = mid + 1; else hi = mid;
+    }
+    s_h1 = lo;
+  }
+  __syncthreads();
+
+  while (true) {
+    if (*(volatile int*)&va.flags[0] == 0 || *(volatile int*)&va.flags[3] != 0) break;
+    // ---------------- A: Ap = L_eps p on own rows, p.Ap
+    float2 dot[VPL][4];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
+    for (int64_t h = s_h0; h < s_h1; ++h) {
+      const int64_t u = a.heavy[h];
+      const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+      const int64_t per = (j1 - j0 + GPB - 1) / GPB;
+      const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
+      float4 pu[VPL], acc[VPL];
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
+        acc[v] = f4_zero();
+      }
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, nvec, pu, s0, s1, acc);
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q < nvec) reinterpret_cast<float4*>(comb + gi * ld)[q] = acc[v];
+      }
+      __syncthreads();
+      if (gi == 0) {
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int q = gl + LPR * v;
+          if (q >= nvec) continue;
+          float4 s = f4_zero();
+          for (int g = 0; g < GPB; ++g) {
+            const float4 c = reinterpret_cast<const float4*>(comb + g * ld)[q];
+            s.x += c.x;
+            s.y += c.y;
+            s.z += c.z;
+            s.w += c.w;
+          }
+          float4 o;
+          o.x = fmaf(a.eps, pu[v].x, s.x);
+          o.y = fmaf(a.eps, pu[v].y, s.y);
+          o.z = fmaf(a.eps, pu[v].z, s.z);
+          o.w = fmaf(a.eps, pu[v].w, s.w);
+          reinterpret_cast<float4*>(aps + (size_t)(u - r0) * ld)[q] = o;
+          dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
+          dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
+          dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
+          dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
+        }
+      }
+      __syncthreads();
+    }
+    for (int i = gi; i < nrows; i += GPB) {
+      const int64_t u = r0 + i;
+      const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+      if (j1 - j0 > a.H) continue;
+      float4 pu[VPL], acc[VPL];
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
+        acc[v] = f4_zero();
+      }
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, nvec, pu, j0, j1, acc);
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q >= nvec) continue;
+        float4 o;
+        o.x = fmaf(a.eps, pu[v].x, acc[v].x);
+        o.y = fmaf(a.eps, pu[v].y, acc[v].y);
+        o.z = fmaf(a.eps, pu[v].z, acc[v].z);
+        o.w = fmaf(a.eps, pu[v].w, acc[v].w);
+        reinterpret_cast<float4*>(aps + (size_t)i * ld)[q] = o;
+        dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
+        dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
+        dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
+        dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
+      }
+    }
+    if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
+    __syncthreads();
+    block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
+    if (grid_colreduce(a.cr, sbuf, sbuf, ld)) {
+      for (int c = threadIdx.x; c < ld; c += PT) {
+        const double v = df_value(sbuf[c]);
+        float al = 0.f;
+        if (*(volatile int*)&va.active[c]) {
+          const double q = *(volatile double*)&va.rr[c] / v;
+          if (!(v > 0.0) || !isfinite(q)) {
+            va.active[c] = 0;
+            atomicOr(&va.flags[1], 1);
+          } else {
+            al = (float)q;
+          }
+        }
+        va.alpha[c] = al;
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        __threadfence();
+        red_release_add(va.gen, 1u);
+      }
+    } else {
+      wait_generation(va.gen, s_gen, va.flags);
+    }
+    __syncthreads();
+
+    // ---------------- B: x += alpha p, r -= alpha Ap, r.r
+    float4 al[VPL];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      al[v] = q < nvec ? ldcg_f4(va.alpha + 4 * q) : f4_zero();
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; ++v)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
+    for (int i = gi; i < nrows; i += GPB) {
+      const size_t ig = (size_t)(r0 + i) * ld;
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q >= nvec) continue;
+        const float4 p = ldcg_f4(a.P + ig + 4 * q);
+        float4 x = *reinterpret_cast<const float4*>(va.X + ig + 4 * q);
+        float4 r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
+        const float4 ap = reinterpret_cast<const float4*>(aps + (size_t)i * ld)[q];
+        x.x = fmaf(al[v].x, p.x, x.x);
+        x.y = fmaf(al[v].y, p.y, x.y);
+        x.z = fmaf(al[v].z, p.z, x.z);
+        x.w = fmaf(al[v].w, p.w, x.w);
+        r.x = fmaf(-al[v].x, ap.x, r.x);
+        r.y = fmaf(-al[v].y, ap.y, r.y);
+        r.z = fmaf(-al[v].z, ap.z, r.z);
+        r.w = fmaf(-al[v].w, ap.w, r.w);
+        *reinterpret_cast<float4*>(va.X + ig + 4 * q) = x;
+        reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = r;
+        dot[v][0] = df_fma(dot[v][0], r.x, r.x);
+        dot[v][1] = df_fma(dot[v][1], r.y, r.y);
+        dot[v][2] = df_fma(dot[v][2], r.z, r.z);
+        dot[v][3] = df_fma(dot[v][3], r.w, r.w);
+      }
+    }
+    if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
+    __syncthreads();
+    block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
+    if (grid_colreduce(a.cr, sbuf, sbuf, ld)) {
+      int any = 0;
+      for (int c = threadIdx.x; c < ld; c += PT) {
+        float be = 0.f;
+        int act = *(volatile int*)&va.active[c];
+        if (act) {
+          const double rn = df_value(sbuf[c]);
+          const int it = *(volatile int*)&va.iters[c] + 1;
+          va.iters[c] = it;
+          if (!isfinite(rn)) {
+            act = 0;
+            atomicOr(&va.flags[1], 1);
+          } else {
+            be = (float)(rn / *(volatile double*)&va.rr[c]);
+            va.rr[c] = rn;
+            if (rn <= va.tol2 * *(volatile double*)&va.yy[c]) {
+              va.conv[c] = 1;
+              act = 0;
+            } else if (it >= va.max_iter) {
+              act = 0;
+            }
+          }
+          va.active[c] = act;
+        }
+        va.beta[c] = be;
+        any |= act;
+      }
+      any = __syncthreads_or(any);
+      if (threadIdx.x == 0) {
+        va.flags[0] = any;
+        __threadfence();
+        red_release_add(va.gen, 1u);
+      }
+    } else {
+      wait_generation(va.gen, s_gen, va.flags);
+    }
+    __syncthreads();
+
+    // ---------------- C: p = r + beta p on active columns
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q >= nvec) continue;
+      const int4 act = __ldcg(reinterpret_cast<const int4*>(va.active + 4 * q));
+      if (!(act.x | act.y | act.z | act.w)) continue;
+      const float4 be = ldcg_f4(va.beta + 4 * q);
+      for (int i = gi; i < nrows; i += GPB) {
+        const size_t ig = (size_t)(r0 + i) * ld + 4 * q;
+        const float4 r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
+        float4 p = ldcg_f4(a.P + ig);
+        if (act.x) p.x = fmaf(be.x, p.x, r.x);
+        if (act.y) p.y = fmaf(be.y, p.y, r.y);
+        if (act.z) p.z = fmaf(be.z, p.z, r.z);
+        if (act.w) p.w = fmaf(be.w, p.w, r.w);
+        *reinterpret_cast<float4*>(const_cast<float*>(a.P) + ig) = p;
+      }
+    }
+    grid_barrier(bar_cnt, va.gen, va.flags);
+  }
+}
+
 // ---------------------------------------------------------------------------- heavy rows
 __global__ void k_mark_heavy(const int64_t* __restrict__ row_ptr, int32_t n, int32_t H,
                              uint8_t* __restrict__ flag) {
@@ -617,6 +954,71 @@ erc_status launch_update(const VecArgs& va, int grid, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   ERC_CUDA(cudaLaunchKernelEx(&cfg, k_update_fused, va));
+  count_launches(1);
+  return ERC_OK;
+}
+
+// ---- resident path selection: the kernel for this shape, its shared memory, and whether it fits
+const void* resident_kernel(int nvec, bool weighted) {
+  const void* k = nullptr;
+  auto pick = [&](auto lpr, auto vpl) {
+    constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
+    k = weighted ? (const void*)k_cg_resident<LPR, VPL, true>
+                 : (const void*)k_cg_resident<LPR, VPL, false>;
+  };
+  if (nvec <= 4) pick(ic<4>{}, ic<1>{});
+  else if (nvec <= 8) pick(ic<8>{}, ic<1>{});
+  else if (nvec <= 16) pick(ic<16>{}, ic<1>{});
+  else if (nvec <= 32) pick(ic<32>{}, ic<1>{});
+  else if (nvec <= 64) pick(ic<32>{}, ic<2>{});
+  return k;  // wider rows use the multi-kernel path
+}
+
+bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const void** kern) {
+  const char* mode = getenv("ERC_CG_MODE");
+  if (mode && strcmp(mode, "graph") == 0) return false;
+  const int nvec = ld / 4;
+  const void* k = resident_kernel(nvec, g->val != nullptr);
+  if (!k) return false;
+  const int lpr = nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32;
+  const int grid = sm_count();
+  const int64_t rows = ((int64_t)g->n + grid - 1) / grid;
+  const size_t bytes = 4 * (2 * (size_t)rows * ld + (size_t)(PT / lpr) * ld + 2 * (size_t)ld +
+                            2 * (size_t)PWARPS * PCH);
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    return false;
+  if (bytes > (size_t)optin) return false;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  int nb = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, PT, bytes) != cudaSuccess || nb < 1) {
+    cudaGetLastError();
+    return false;
+  }
+  *rb = (int32_t)rows;
+  *smem = bytes;
+  *kern = k;
+  return true;
+}
+
+erc_status launch_resident(const void* kern, const ResArgs& ra, size_t smem, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sm_count());
+  cfg.blockDim = dim3(PT);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;  // one block per SM, all resident
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  void* args[] = {const_cast<ResArgs*>(&ra)};
+  ERC_CUDA(cudaLaunchKernelExC(&cfg, kern, args));
   count_launches(1);
   return ERC_OK;
 }
@@ -817,18 +1219,27 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
 
-  const int S = iterations_per_poll(g, ld);
-  cudaGraphExec_t exec = nullptr;
-  ERC_TRY(iteration_graph(sa, sgrid, va, ugrid, S, &exec));
-  int done = 0;
-  int h_any = 1;
-  while (done < max_iter) {
-    ERC_CUDA(cudaGraphLaunch(exec, s));
-    count_launches(2LL * S);  // the graph holds S iterations of two kernels
-    done += S;
-    ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
-    ERC_CUDA(cudaStreamSynchronize(s));
-    if (!h_any) break;
+  int32_t rb = 0;
+  size_t smem = 0;
+  const void* kres = nullptr;
+  if (resident_plan(g, ld, &rb, &smem, &kres)) {
+    // the whole solve in one cooperative launch, no host round trips
+    ResArgs ra{sa, va, rb};
+    ERC_TRY(launch_resident(kres, ra, smem, s));
+  } else {
+    const int S = iterations_per_poll(g, ld);
+    cudaGraphExec_t exec = nullptr;
+    ERC_TRY(iteration_graph(sa, sgrid, va, ugrid, S, &exec));
+    int done = 0;
+    int h_any = 1;
+    while (done < max_iter) {
+      ERC_CUDA(cudaGraphLaunch(exec, s));
+      count_launches(2LL * S);  // the graph holds S iterations of two kernels
+      done += S;
+      ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
+      ERC_CUDA(cudaStreamSynchronize(s));
+      if (!h_any) break;
+    }
   }
 
   // true residual of the returned iterate, plus the per-column outputs

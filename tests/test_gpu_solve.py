@@ -45,6 +45,31 @@ def test_cg_matches_oracle_cg(kc):
     assert np.all(host(X)[:, kc:] == 0)
 
 
+@pytest.mark.parametrize("mode", ["graph", "auto"])
+@pytest.mark.parametrize("kc,weighted,heavy", [(16, True, False), (128, False, False),
+                                               (64, True, True), (256, False, False)])
+def test_cg_paths_match_oracle(monkeypatch, mode, kc, weighted, heavy):
+    """The multi-kernel path and the resident single-launch path against the oracle."""
+    monkeypatch.setenv("ERC_CG_MODE", mode)
+    n, src, dst, w = synth.random_connected(4000, 16000, seed=kc, weighted=weighted)
+    if heavy:  # attach a hub to 3000 nodes so the block-split rows are exercised
+        hub_dst = np.arange(1, 3001, dtype=np.int32)
+        src = np.concatenate([src, np.zeros(3000, np.int32)])
+        dst = np.concatenate([dst, hub_dst])
+        if w is not None:
+            w = np.concatenate([w, np.full(3000, 0.75, np.float32)])
+    g, ref = build_both(n, src, dst, w)
+    Y = erc.erc_jl_rhs(g, 9, 256, 0, kc)
+    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, kc, 1e-6)
+    assert st == erc.ERC_OK
+    Xr, itr, _, _ = O.batched_cg(ref, 1e-3, O.jl_rhs(ref, 9, 256, 0, kc), 1e-6)
+    Rg = torch.zeros(g.m, device=dev())
+    erc.erc_edge_resistance(g, X, kc, Rg)
+    _check_R(host(Rg), O.edge_resistance(ref, Xr))
+    assert np.all(np.abs(host(iters) - itr) <= 0.1 * itr + 2)
+    assert np.all(host(relres) <= 2e-6)
+
+
 def test_cg_not_converged_and_zero_columns():
     n, src, dst, w = synth.random_connected(1000, 3000, seed=5)
     g, ref = build_both(n, src, dst, w)
