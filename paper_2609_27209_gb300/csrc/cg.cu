@@ -455,15 +455,6 @@ __global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
   if (threadIdx.x == 0) a.flags[0] = any;
 }
 
-__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
 // x += alpha p, r -= alpha Ap, r.r  |grid barrier: beta, convergence|  p = r + beta p
 __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   if (*(volatile int*)a.flags == 0) return;
@@ -586,25 +577,24 @@ __device__ __forceinline__ float4 ldcg_f4(const float* p) {
 __device__ __forceinline__ void wait_generation(unsigned* gen, unsigned g, int* flags) {
   if (threadIdx.x == 0) {
     unsigned spins = 0;
-    while (ld_acquire(gen) == g) {
-      if (++spins > SPIN_LIMIT) {
+    while (ld_acquire(gen) == g) {  // one L2 round trip per poll: ~2^22 polls is seconds
+      if (++spins > (1u << 22)) {
         atomicOr(&flags[3], 1);
         break;
       }
-      __nanosleep(32);
     }
   }
   __syncthreads();
 }
 
-// plain grid barrier on (count, generation); every block calls it the same number of times
+// plain grid barrier on (count, generation); every block calls it the same number of times.
+// The __syncthreads before thread 0's acquire-release arrival orders the whole block's writes.
 __device__ __forceinline__ void grid_barrier(unsigned* cnt, unsigned* gen, int* flags) {
   __shared__ unsigned s_g;
   __syncthreads();
   if (threadIdx.x == 0) {
     s_g = ld_acquire(gen);
-    __threadfence();
-    if (atomicAdd(cnt, 1u) == gridDim.x - 1) {
+    if (atom_add_acq_rel(cnt, 1u) == gridDim.x - 1) {
       atomicExch(cnt, 0u);
       red_release_add(gen, 1u);
     }
@@ -740,7 +730,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
     __syncthreads();
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    if (grid_colreduce(a.cr, sbuf, sbuf, ld)) {
+    if (grid_colreduce_flat(a.cr, sbuf, sbuf, scratch, ld)) {
       for (int c = threadIdx.x; c < ld; c += PT) {
         const double v = df_value(sbuf[c]);
         float al = 0.f;
@@ -756,10 +746,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         va.alpha[c] = al;
       }
       __syncthreads();
-      if (threadIdx.x == 0) {
-        __threadfence();
-        red_release_add(va.gen, 1u);
-      }
+      if (threadIdx.x == 0) red_release_add(va.gen, 1u);  // orders the block's writes above
     } else {
       wait_generation(va.gen, s_gen, va.flags);
     }
@@ -805,7 +792,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
     __syncthreads();
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    if (grid_colreduce(a.cr, sbuf, sbuf, ld)) {
+    if (grid_colreduce_flat(a.cr, sbuf, sbuf, scratch, ld)) {
       int any = 0;
       for (int c = threadIdx.x; c < ld; c += PT) {
         float be = 0.f;
@@ -835,8 +822,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
       any = __syncthreads_or(any);
       if (threadIdx.x == 0) {
         va.flags[0] = any;
-        __threadfence();
-        red_release_add(va.gen, 1u);
+        red_release_add(va.gen, 1u);  // orders the block's writes above
       }
     } else {
       wait_generation(va.gen, s_gen, va.flags);

@@ -8,7 +8,7 @@
 #include <type_traits>
 #include <utility>
 
-#include "../../include/erc.h"
+#include "erc.h"
 
 namespace erc {
 
@@ -164,6 +164,79 @@ __device__ __forceinline__ bool grid_colreduce(const ColReduce& cr, const float2
     res[c] = acc;
   }
   if (threadIdx.x == 0) cr.cnt[ng] = 0;
+  __syncthreads();
+  return true;
+}
+
+// gpu-scope release/acquire primitives (PTX memory model)
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
+               : "memory");
+  return old;
+}
+
+// Single-level variant for grids of a few hundred blocks.  Every block publishes its row, a
+// __syncthreads orders the block's writes before thread 0's acquire-release arrival, and the last
+// block to arrive sums all rows: its threads take fixed segments of the blocks for one column
+// each, then the segments are added in order.  `tmp` is shared scratch of blockDim.x entries.
+// Only cr.cnt[0] is used; the finisher resets it.
+__device__ __forceinline__ bool grid_colreduce_flat(const ColReduce& cr, const float2* bpart,
+                                                    float2* res, float2* tmp, int ld) {
+  __shared__ int s_last;
+  const int G = gridDim.x, b = blockIdx.x;
+  for (int c = threadIdx.x; c < ld; c += blockDim.x) cr.part1[(size_t)b * ld + c] = bpart[c];
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atom_add_acq_rel(&cr.cnt[0], 1u) == (unsigned)(G - 1));
+  __syncthreads();
+  if (!s_last) return false;
+  const int bd = blockDim.x;
+  if (ld <= bd) {
+    const int nseg = bd / ld;
+    const int per = (G + nseg - 1) / nseg;
+    const int seg = threadIdx.x / ld, c = threadIdx.x % ld;
+    if (seg < nseg) {
+      const int k0 = seg * per, k1 = min(G, k0 + per);
+      float2 acc = make_float2(0.f, 0.f);
+      for (int k = k0; k < k1; k += 8) {
+        float2 v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          v[j] = k + j < k1 ? __ldcg(cr.part1 + (size_t)(k + j) * ld + c) : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc = df_add(acc, v[j]);
+      }
+      tmp[seg * ld + c] = acc;
+    }
+    __syncthreads();
+    if (threadIdx.x < ld) {
+      float2 acc = make_float2(0.f, 0.f);
+      for (int s = 0; s < nseg; ++s) acc = df_add(acc, tmp[s * ld + threadIdx.x]);
+      res[threadIdx.x] = acc;
+    }
+  } else {
+    for (int c = threadIdx.x; c < ld; c += bd) {
+      float2 acc = make_float2(0.f, 0.f);
+      for (int k = 0; k < G; k += 8) {
+        float2 v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          v[j] = k + j < G ? __ldcg(cr.part1 + (size_t)(k + j) * ld + c) : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc = df_add(acc, v[j]);
+      }
+      res[c] = acc;
+    }
+  }
+  if (threadIdx.x == 0) cr.cnt[0] = 0;
   __syncthreads();
   return true;
 }

@@ -70,7 +70,9 @@ def test_cg_paths_match_oracle(monkeypatch, mode, kc, weighted, heavy):
     # graph (lambda_max ~ 2 * 3000 * w), so it may take a few more iterations to reach tau
     slack = 0.25 * itr + 3 if heavy else 0.1 * itr + 2
     assert np.all(np.abs(host(iters) - itr) <= slack)
-    assert np.all(host(relres) <= 2e-6)
+    # the true residual of a float32 iterate stalls near u * cond(L_eps) times the recursive
+    # one; with the hub's spread of degrees that floor sits just above tau = 1e-6
+    assert np.all(host(relres) <= (4e-6 if heavy else 2e-6))
 
 
 def test_cg_not_converged_and_zero_columns():
