@@ -164,6 +164,28 @@ erc_status erc_sampling_probs(const erc_graph* g, const float* kappa, float eta,
                               float* prob_edge, void* ws, size_t ws_bytes, erc_stream s);
 
 /* ---------------------------------------------------------------------------------------------
+ * erc_sampling_probs_noalloc -- erc_sampling_probs with no caller workspace and no allocation.
+ *
+ * The paper has no counterpart; this is a library convenience.  It serves callers that cannot
+ * allocate device memory themselves: plug-ins whose host application owns every device buffer,
+ * code that must not call cudaMalloc / cudaFree because those calls can synchronise the whole
+ * device, and processes held to a fixed device-memory budget.  Inputs and outputs are as for
+ * erc_sampling_probs; the scratch is a file-scope device array of
+ * ERC_SAMPLING_PROBS_NOALLOC_SCRATCH_BYTES inside liberc.so, present on every device that loads
+ * the library and held until the process exits.  The call allocates nothing.
+ * Limits: g->n <= ERC_SAMPLING_PROBS_NOALLOC_MAX_NODES, else ERC_ERR_CAPACITY (nothing is run).
+ * The first call on each device looks up the array's device address (cudaGetSymbolAddress) with
+ * that device current; make that first call before any stream capture.  All calls share the one
+ * array and it keeps the last call's contents (a call never relies on them): calls that may
+ * overlap on the GPU -- concurrent streams, or several host threads -- race with each other and
+ * must be serialised by the caller.
+ * ------------------------------------------------------------------------------------------- */
+#define ERC_SAMPLING_PROBS_NOALLOC_MAX_NODES 4000000
+#define ERC_SAMPLING_PROBS_NOALLOC_SCRATCH_BYTES (32u << 20)
+erc_status erc_sampling_probs_noalloc(const erc_graph* g, const float* kappa, float eta,
+                                      float* prob_node, float* prob_edge, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
  * erc_laplacian_apply -- AP = L_eps P for an n x ld block (the CG operator of Eq. 5), and, when
  * pAp is not NULL, pAp[c] = sum_u P[u,c] AP[u,c] as float64 (device [kc]).  Exposed for testing
  * and benchmarking the operator alone.

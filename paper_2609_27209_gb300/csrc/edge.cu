@@ -3,6 +3,7 @@
 //   erc_curvature        p_u = 1 - 1/2 sum_v w_uv R_uv, kappa_uv = 2 (p_u + p_v) / R_uv (Eq. 2)
 //   erc_sampling_probs   Eq. 7 (with the uniform fallback), Eq. 8, normalisation (§3.2)
 #include <cfloat>
+#include <mutex>
 
 #include "erc_internal.cuh"
 
@@ -365,4 +366,59 @@ extern "C" erc_status erc_sampling_probs(const erc_graph* g, const float* kappa,
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
+}
+
+// ------------------------------------------------------------------------------------------------
+// erc_sampling_probs_noalloc: erc_sampling_probs for callers that cannot allocate device memory.
+// Its scratch is this file-scope device array instead of a caller workspace.  The array exists on
+// every device that loads the library and stays allocated until the process exits.
+// ------------------------------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_probs_noalloc_scratch[ERC_SAMPLING_PROBS_NOALLOC_SCRATCH_BYTES];
+
+namespace erc {
+namespace {
+// The array's device address, looked up once per device with that device current.  In host code
+// the symbol names a host-side stand-in, never the device memory, so kernels only ever receive
+// this looked-up address.
+erc_status noalloc_scratch(void** out) {
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  ERC_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) return set_error(ERC_ERR_CUDA, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_probs_noalloc_scratch);
+    if (e != cudaSuccess || !p)
+      return set_error(ERC_ERR_CUDA, "cudaGetSymbolAddress(scratch) failed on device %d: %s",
+                       dev, cudaGetErrorString(e));
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return ERC_OK;
+}
+}  // namespace
+}  // namespace erc
+
+extern "C" erc_status erc_sampling_probs_noalloc(const erc_graph* g, const float* kappa,
+                                                 float eta, float* prob_node, float* prob_edge,
+                                                 erc_stream stream) {
+  clear_error();
+  ERC_TRY(check_graph(g));
+  if (g->n > ERC_SAMPLING_PROBS_NOALLOC_MAX_NODES)
+    return set_error(ERC_ERR_CAPACITY,
+                     "erc_sampling_probs_noalloc handles at most %d nodes (got %d); use "
+                     "erc_sampling_probs with a caller workspace",
+                     ERC_SAMPLING_PROBS_NOALLOC_MAX_NODES, g->n);
+  const size_t need = erc_sampling_probs_workspace_size(g->n, g->m);
+  if (need > sizeof(g_probs_noalloc_scratch))
+    return set_error(ERC_ERR_CAPACITY, "scratch needs %zu bytes, the static array holds %zu",
+                     need, sizeof(g_probs_noalloc_scratch));
+  void* scratch = nullptr;
+  ERC_TRY(noalloc_scratch(&scratch));
+  // every word of the scratch that this call reads is written earlier in the same call, so the
+  // previous call's leftovers need no clearing
+  return erc_sampling_probs(g, kappa, eta, prob_node, prob_edge, scratch,
+                            sizeof(g_probs_noalloc_scratch), stream);
 }

@@ -66,6 +66,8 @@ _SIGS = {
     "erc_sampling_probs_workspace_size": (_sz, [_i32, _i64]),
     "erc_sampling_probs": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _f32, _c_p, _c_p, _c_p, _sz,
                                   _c_p]),
+    "erc_sampling_probs_noalloc": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _f32, _c_p, _c_p,
+                                          _c_p]),
     "erc_laplacian_apply_workspace_size": (_sz, [_i32, _i32]),
     "erc_laplacian_apply": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _c_p,
                                    _c_p, _sz, _c_p]),
@@ -236,6 +238,23 @@ def erc_sampling_probs(g, kappa, eta=1e-8):
     gc = g.c()
     _check(lib().erc_sampling_probs(ctypes.byref(gc), _ptr(kappa), eta, _ptr(pn), _ptr(pe),
                                     _ptr(ws), ws.numel(), _stream()))
+    return pn, pe
+
+
+def erc_sampling_probs_noalloc(g, kappa, eta=1e-8, out=None):
+    """erc_sampling_probs without a workspace: the library's static device scratch is used.
+
+    For callers that cannot allocate device memory; pass preallocated `out` = (prob_node,
+    prob_edge) to keep the call itself free of allocations on the Python side too.
+    """
+    dev = kappa.device
+    if out is None:
+        out = (torch.empty(g.n, dtype=torch.float32, device=dev),
+               torch.empty(max(g.m, 1), dtype=torch.float32, device=dev)[:g.m])
+    pn, pe = out
+    gc = g.c()
+    _check(lib().erc_sampling_probs_noalloc(ctypes.byref(gc), _ptr(kappa), eta, _ptr(pn),
+                                            _ptr(pe), _stream()))
     return pn, pe
 
 
