@@ -133,6 +133,15 @@ erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* 
                           int32_t kc, float tol, int32_t max_iter, int32_t* iters, float* relres,
                           void* ws, size_t ws_bytes, erc_stream s);
 
+/* erc_batched_cg_timed -- benchmarking helper: erc_batched_cg, plus *solve_us (host) = the time
+ * between CUDA events recorded on `s` around the iteration kernels (initialisation and the final
+ * residual excluded) and *path (host) = 1 when the single-launch resident solver ran, 0 for the
+ * multi-kernel path (graphs whose r and Ap blocks exceed the SMs' shared memory). */
+erc_status erc_batched_cg_timed(const erc_graph* g, float eps, const float* Y, float* X,
+                                int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                float* solve_us, int32_t* path, erc_stream s);
+
 /* ---------------------------------------------------------------------------------------------
  * erc_edge_resistance -- R_acc[e] += sum_{c < kc} (X[eu[e], c] - X[ev[e], c])^2   (Eq. 6).
  *

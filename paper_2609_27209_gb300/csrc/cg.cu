@@ -1124,11 +1124,10 @@ extern "C" size_t erc_batched_cg_workspace_size(int32_t n, int32_t ld) {
   return a.used + 256;
 }
 
-extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* X,
-                                     int32_t ld, int32_t kc, float tol, int32_t max_iter,
-                                     int32_t* iters, float* relres, void* ws, size_t ws_bytes,
-                                     erc_stream stream) {
-  clear_error();
+static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y, float* X,
+                                  int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                  int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                  erc_stream stream, float* solve_us, int32_t* path) {
   ERC_TRY(check_graph(g));
   ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
   ERC_REQUIRE(eps > 0.f && isfinite(eps), "eps must be positive");
@@ -1208,7 +1207,15 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   int32_t rb = 0;
   size_t smem = 0;
   const void* kres = nullptr;
-  if (resident_plan(g, ld, &rb, &smem, &kres)) {
+  const bool resident = resident_plan(g, ld, &rb, &smem, &kres);
+  if (path) *path = resident ? 1 : 0;
+  cudaEvent_t ev[2] = {nullptr, nullptr};
+  if (solve_us) {
+    ERC_CUDA(cudaEventCreate(&ev[0]));
+    ERC_CUDA(cudaEventCreate(&ev[1]));
+    ERC_CUDA(cudaEventRecord(ev[0], s));
+  }
+  if (resident) {
     // the whole solve in one cooperative launch, no host round trips
     ResArgs ra{sa, va, rb};
     ERC_TRY(launch_resident(kres, ra, smem, s));
@@ -1227,6 +1234,7 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
       if (!h_any) break;
     }
   }
+  if (solve_us) ERC_CUDA(cudaEventRecord(ev[1], s));
 
   // true residual of the returned iterate, plus the per-column outputs
   SpmmArgs ra = sa;
@@ -1235,12 +1243,40 @@ extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float*
   int h_flags[4] = {0, 0, 0, 0};
   ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 4 * sizeof(int), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
+  if (solve_us) {
+    float ms = 0.f;
+    const cudaError_t e = cudaEventElapsedTime(&ms, ev[0], ev[1]);
+    cudaEventDestroy(ev[0]);
+    cudaEventDestroy(ev[1]);
+    if (e != cudaSuccess) return set_error(ERC_ERR_CUDA, "event timing: %s", cudaGetErrorString(e));
+    *solve_us = 1000.f * ms;
+  }
   if (h_flags[3]) return set_error(ERC_ERR_TIMEOUT, "update kernel grid barrier timed out");
   if (h_flags[1]) return set_error(ERC_ERR_NUMERIC, "non-finite or non-positive CG scalar");
   if (h_flags[2])
     return set_error(ERC_ERR_NOT_CONVERGED, "%d of %d columns reached max_iter=%d", h_flags[2],
                      kc, max_iter);
   return ERC_OK;
+}
+
+extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* X,
+                                     int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                     int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                     erc_stream stream) {
+  clear_error();
+  return batched_cg_impl(g, eps, Y, X, ld, kc, tol, max_iter, iters, relres, ws, ws_bytes, stream,
+                         nullptr, nullptr);
+}
+
+extern "C" erc_status erc_batched_cg_timed(const erc_graph* g, float eps, const float* Y,
+                                           float* X, int32_t ld, int32_t kc, float tol,
+                                           int32_t max_iter, int32_t* iters, float* relres,
+                                           void* ws, size_t ws_bytes, float* solve_us,
+                                           int32_t* path, erc_stream stream) {
+  clear_error();
+  ERC_REQUIRE(solve_us && path, "solve_us and path are required");
+  return batched_cg_impl(g, eps, Y, X, ld, kc, tol, max_iter, iters, relres, ws, ws_bytes, stream,
+                         solve_us, path);
 }
 
 extern "C" size_t erc_laplacian_apply_workspace_size(int32_t n, int32_t ld) {

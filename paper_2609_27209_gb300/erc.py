@@ -61,6 +61,9 @@ _SIGS = {
     "erc_batched_cg_workspace_size": (_sz, [_i32, _i32]),
     "erc_batched_cg": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _f32,
                               _i32, _c_p, _c_p, _c_p, _sz, _c_p]),
+    "erc_batched_cg_timed": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32,
+                                    _f32, _i32, _c_p, _c_p, _c_p, _sz, ctypes.POINTER(_f32),
+                                    ctypes.POINTER(_i32), _c_p]),
     "erc_edge_resistance": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _i32, _i32, _c_p, _c_p]),
     "erc_curvature": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _c_p, _c_p, _c_p]),
     "erc_sampling_probs_workspace_size": (_sz, [_i32, _i64]),
@@ -212,6 +215,25 @@ def erc_batched_cg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
                                      max_iter, _ptr(iters), _ptr(relres), _ptr(ws), ws.numel(),
                                      _stream()), allow=(ERC_ERR_NOT_CONVERGED,))
     return X, iters, relres, st
+
+
+def erc_batched_cg_timed(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
+    """erc_batched_cg plus (solve microseconds, path): path 1 = resident single-launch solver."""
+    n, ld = Y.shape
+    dev = Y.device
+    X = torch.empty_like(Y) if X is None else X
+    iters = torch.empty(kc, dtype=torch.int32, device=dev)
+    relres = torch.empty(kc, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = _workspace(lib().erc_batched_cg_workspace_size(n, ld), dev)
+    us = _f32(0)
+    path = _i32(0)
+    gc = g.c()
+    st = _check(lib().erc_batched_cg_timed(ctypes.byref(gc), eps, _ptr(Y), _ptr(X), ld, kc, tol,
+                                           max_iter, _ptr(iters), _ptr(relres), _ptr(ws),
+                                           ws.numel(), ctypes.byref(us), ctypes.byref(path),
+                                           _stream()), allow=(ERC_ERR_NOT_CONVERGED,))
+    return X, iters, relres, st, float(us.value), int(path.value)
 
 
 def erc_edge_resistance(g, X, kc, R_acc):
