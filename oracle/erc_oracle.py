@@ -176,17 +176,20 @@ def jl_q(seed, K, e, c0, kc):
     return (1.0 - 2.0 * bits.astype(np.float64)) / np.sqrt(K)
 
 
-def jl_rhs(g, seed, K, c0, kc, edge_block=1 << 16):
+def jl_rhs(g, seed, K, c0, kc, edge_block=1 << 16, edge_ids=None):
     """Y = B^T W^{1/2} Q[:, c0:c0+kc]  (n x kc, float64), streamed over blocks of edges (§3.1.2).
 
     Edge e adds +sqrt(w_e) Q[e, :] to row eu[e] and -sqrt(w_e) Q[e, :] to row ev[e].
+    `edge_ids` (optional) gives the id each edge of `g` has in a larger graph, so that rows of a
+    subgraph holding every edge of those rows reproduce the larger graph's Y on them.
     """
     n, m = g["n"], g["m"]
     Y = np.zeros((n, kc))
     sw = np.sqrt(g["ew"].astype(np.float64))
+    ids = np.arange(m) if edge_ids is None else np.asarray(edge_ids, dtype=np.int64)
     for e0 in range(0, m, edge_block):
         e = np.arange(e0, min(m, e0 + edge_block))
-        V = sw[e, None] * jl_q(seed, K, e, c0, kc)
+        V = sw[e, None] * jl_q(seed, K, ids[e], c0, kc)
         np.add.at(Y, g["eu"][e], V)
         np.add.at(Y, g["ev"][e], -V)
     return Y

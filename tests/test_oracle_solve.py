@@ -91,3 +91,17 @@ def test_cg_stops_columns_independently():
         x1, it1, _, _ = O.batched_cg(g, 1e-3, Y[:, c:c + 1], 1e-6)
         assert it1[0] == iters[c]
         np.testing.assert_allclose(X[:, c], x1[:, 0], rtol=1e-12, atol=1e-15)
+
+
+def test_rhs_rows_of_a_subgraph_with_global_edge_ids():
+    """Rows whose every edge is in a subgraph get the full graph's Y when edges keep their ids."""
+    n, src, dst, w = synth.random_connected(300, 1200, seed=12)
+    g = O.build_laplacian(n, src, dst, w)
+    Y = O.jl_rhs(g, 7, 96, 32, 40)
+    S = np.array([0, 5, 17, 123, 299])
+    keep = np.isin(src, S) | np.isin(dst, S)
+    sub = O.build_laplacian(n, src[keep], dst[keep], w[keep])
+    keys = g["eu"].astype(np.int64) * n + g["ev"]
+    ids = np.searchsorted(keys, sub["eu"].astype(np.int64) * n + sub["ev"])
+    Ys = O.jl_rhs(sub, 7, 96, 32, 40, edge_ids=ids)
+    np.testing.assert_allclose(Ys[S], Y[S], rtol=0, atol=1e-14)
