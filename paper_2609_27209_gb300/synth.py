@@ -66,6 +66,18 @@ def _keys(u, v, n):
     return a * n + b
 
 
+def _unique_sorted(k):
+    """Sorted distinct values (a sort and a neighbour compare: much faster than np.unique's
+    hashing path on tens of millions of int64 keys, same result)."""
+    k = np.sort(np.asarray(k, dtype=np.int64))
+    if k.size == 0:
+        return k
+    keep = np.empty(k.size, dtype=bool)
+    keep[0] = True
+    np.not_equal(k[1:], k[:-1], out=keep[1:])
+    return k[keep]
+
+
 def _ring_keys(n):
     i = np.arange(n, dtype=np.int64)
     return _keys(i, (i + 1) % n, n)
@@ -73,7 +85,7 @@ def _ring_keys(n):
 
 def _finish(rng, n, keys, weights="unit", sigma=0.5):
     """Sorted unique canonical keys -> shuffled, randomly oriented (n, src, dst, w)."""
-    keys = np.unique(keys)
+    keys = _unique_sorted(keys)
     m = keys.size
     if weights == "unit":
         w = None
@@ -105,7 +117,7 @@ def _draw_distinct(rng, count, draw_batch, n, exclude=None):
         k = _keys(u[ok], v[ok], n)
         if exclude is not None:
             k = k[~np.isin(k, exclude)]
-        have = np.unique(np.concatenate([have, k]))
+        have = _unique_sorted(np.concatenate([have, k]))
     if have.size > count:
         have = np.sort(rng.choice(have, size=count, replace=False))
     return have
@@ -164,17 +176,38 @@ def chung_lu_weights(n, gamma, mean_deg):
     return np.minimum(s * base, np.sqrt(w.sum()))
 
 
+def alias_table(p):
+    """Walker / Vose alias table of a discrete distribution p (sums to 1): (prob, alias)."""
+    n = p.size
+    q = np.asarray(p, dtype=np.float64) * n
+    prob = np.ones(n)
+    alias = np.arange(n, dtype=np.int64)
+    small = np.nonzero(q < 1.0)[0].tolist()
+    large = np.nonzero(q >= 1.0)[0].tolist()
+    while small and large:
+        s = small.pop()
+        l = large.pop()
+        prob[s] = q[s]
+        alias[s] = l
+        q[l] = (q[l] + q[s]) - 1.0
+        (small if q[l] < 1.0 else large).append(l)
+    return prob, alias
+
+
+def alias_draw(rng, prob, alias, k):
+    """k independent draws from the table's distribution."""
+    i = rng.integers(0, prob.size, k)
+    return np.where(rng.random(k) < prob[i], i, alias[i])
+
+
 def chung_lu(n, gamma, m_target, weights, seed):
     """Chung-Lu power-law graph with `m_target` distinct edges, then a ring added for connectivity."""
     rng = np.random.default_rng(seed)
     wexp = chung_lu_weights(n, gamma, 2.0 * m_target / n)
-    cdf = np.cumsum(wexp)
-    cdf /= cdf[-1]
+    prob, alias = alias_table(wexp / wexp.sum())
 
     def draw(k):
-        u = np.searchsorted(cdf, rng.random(k), side="right")
-        v = np.searchsorted(cdf, rng.random(k), side="right")
-        return np.minimum(u, n - 1), np.minimum(v, n - 1)
+        return alias_draw(rng, prob, alias, k), alias_draw(rng, prob, alias, k)
 
     body = _draw_distinct(rng, m_target, draw, n)
     return _finish(rng, n, np.concatenate([body, _ring_keys(n)]), weights)
