@@ -118,11 +118,6 @@ def spmm_traffic(workload):
 UPDATE_BYTES_PER_ELEM = 28
 
 
-def resident_traffic(workload):
-    """DRAM bytes per launch of the resident CG kernel from a committed ncu summary, if current."""
-    return _traffic("cg_resident", workload)
-
-
 def _traffic(kernel, workload):
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
@@ -297,8 +292,8 @@ def run_ours(args, world, rank, local_rank):
                "d2h_bytes_per_step": d2h, "ms_per_step": 1000 * statistics.mean(et)}
 
     # ---- roofline of the dominant kernel.  On graphs whose r and Ap blocks fit in shared memory
-    # the whole CG solve is one launch (k_cg_resident): its duration comes from CUDA events the
-    # library records around it on its stream.  Otherwise the operator k_spmm dominates and is
+    # the whole CG solve is one launch (k_cg_cluster over column groups, else k_cg_resident): its
+    # duration comes from CUDA events the library records around it on its stream.  Otherwise the operator k_spmm dominates and is
     # timed alone, back to back as inside the CG loop.  Either way the operator alone is also
     # reported under "spmm".
     roof = None
@@ -316,13 +311,14 @@ def run_ours(args, world, rank, local_rank):
                 "frac": op_bytes / t_spmm / 1e9 / peak, "traffic": spmm_traffic(args.config)}
         erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)  # warm
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
-        if path == 1:
+        if path in (1, 2):
             T = int(it_cg.max().item())
             algo = T * (op_bytes + UPDATE_BYTES_PER_ELEM * n * kc)
             ach = algo / (solve_us * 1e-6) / 1e9
+            kname = "k_cg_cluster" if path == 2 else "k_cg_resident"
             roof = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
-                    "frac": ach / peak, "traffic": resident_traffic(args.config),
-                    "kernel": "k_cg_resident (one launch = whole CG solve of a batch)",
+                    "frac": ach / peak, "traffic": _traffic(kname[2:], args.config),
+                    "kernel": f"{kname} (one launch = whole CG solve of a batch)",
                     "iterations": T, "algorithmic_bytes": algo, "launch_us": solve_us,
                     "peak_source": src_kind}
         else:

@@ -134,9 +134,15 @@ erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* 
                           void* ws, size_t ws_bytes, erc_stream s);
 
 /* erc_batched_cg_timed -- benchmarking helper: erc_batched_cg, plus *solve_us (host) = the time
- * between CUDA events recorded on `s` around the iteration kernels (initialisation and the final
- * residual excluded) and *path (host) = 1 when the single-launch resident solver ran, 0 for the
- * multi-kernel path (graphs whose r and Ap blocks exceed the SMs' shared memory). */
+ * between CUDA events recorded on `s` around the solver kernels (the final residual excluded)
+ * and *path (host), the solver that ran:
+ *   2  one launch of thread-block clusters, each solving a group of 16 columns over all rows
+ *      (graphs whose rows' r and Ap slices fit in the shared memory of a cluster, when a cost
+ *      model favours it over 1: small graphs); the launch also initialises r, p and x;
+ *   1  one cooperative launch over all rows and columns (r and Ap blocks in the SMs' shared
+ *      memory; separate initialisation kernel, not timed);
+ *   0  the multi-kernel loop captured in CUDA graphs (larger graphs).
+ * The environment variable ERC_CG_MODE=cluster|resident|graph restricts the choice. */
 erc_status erc_batched_cg_timed(const erc_graph* g, float eps, const float* Y, float* X,
                                 int32_t ld, int32_t kc, float tol, int32_t max_iter,
                                 int32_t* iters, float* relres, void* ws, size_t ws_bytes,

@@ -178,12 +178,13 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
   }
 }
 
-// acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots.
-// L2ONLY loads p through L2 only: required where p is rewritten within the same launch.
+// acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots
+// q = qb + gl + LPR v < qend.  L2ONLY loads p through L2 only: required where p is rewritten
+// within the same launch.
 template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false>
-__device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int nvec,
-                                             const float4 (&pu)[VPL], int64_t j0, int64_t j1,
-                                             float4 (&acc)[VPL]) {
+__device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int qb,
+                                             int qend, const float4 (&pu)[VPL], int64_t j0,
+                                             int64_t j1, float4 (&acc)[VPL]) {
   constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
   for (int64_t jb = j0; jb < j1; jb += LPR) {
     const int64_t jj = jb + gl;
@@ -210,9 +211,9 @@ __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned
       for (int k = 0; k < U; ++k)
 #pragma unroll
         for (int v = 0; v < VPL; ++v) {
-          const int q = gl + LPR * v;
+          const int q = qb + gl + LPR * v;
           const float* src = a.P + (size_t)cj[k] * a.ld + 4 * q;
-          pv[k][v] = (q < nvec && t + k < cnt)
+          pv[k][v] = (q < qend && t + k < cnt)
                          ? (L2ONLY ? __ldcg(reinterpret_cast<const float4*>(src)) : ld_f4(src))
                          : pu[v];
         }
@@ -301,7 +302,7 @@ __global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(Spm
     const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
     float4 pu[VPL], acc[VPL];
     load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
-    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, nvec, pu, s0, s1, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, 0, nvec, pu, s0, s1, acc);
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
@@ -335,7 +336,7 @@ __global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(Spm
     if (j1 - j0 > a.H) continue;
     float4 pu[VPL], acc[VPL];
     load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
-    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, nvec, pu, j0, j1, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, 0, nvec, pu, j0, j1, acc);
     finish_row<LPR, VPL, MODE>(a, u, gl, nvec, pu, acc, dot);
   }
   if (MODE == MODE_APPLY && a.pap_out == nullptr) return;
@@ -554,14 +555,22 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
 // When r and Ap of every row fit in the SMs' shared memory, one cooperative launch runs the whole
 // solve.  Block b owns rows [b rb, b rb + rb): their r and Ap live in its shared memory, x and p
 // in global memory (p is gathered by other blocks).  Per iteration:
-//   A  Ap = L_eps p for own rows (heavy rows by the whole block), p.Ap   -> reduce, alpha
-//   B  x += alpha p, r -= alpha Ap, r.r                                  -> reduce, beta, stop test
+//   A  Ap = L_eps p on own rows (heavy rows by the whole block), p.Ap    -> reduce: alpha
+//   B  x += alpha p, r -= alpha Ap, r.r                                  -> reduce: beta, stop
 //   C  p = r + beta p                                                    -> barrier
-// Every reduce and barrier is a bounded wait on one generation counter.  Data written by other
-// blocks inside the launch (p, scalars) is read through L2 (ld.global.cg), never through L1.
+// A grid synchronisation is an arrival (a release-add on a counter after the block's partials
+// are written) and a bounded wait until all blocks have arrived.  There is no finishing block:
+// after a reduction every block sums all blocks' partials itself, in the same fixed order, so
+// every block derives the same alpha, beta and stop decisions into its own shared memory.  The
+// counter only grows, so the s-th synchronisation waits for s * gridDim arrivals and needs no
+// reset.  Data written by other blocks inside the launch (p, the partials) is read through L2
+// (ld.global.cg), never through L1.  The vector phases B and C issue the loads of several rows
+// before using any of them.
 constexpr int PT = 512;
 constexpr int PWARPS = PT / 32;
 constexpr int PCH = 64;
+constexpr int RMAXLD = 256;  // widest row block the resident kernel takes (64 float4)
+constexpr int RU = 2;  // float4 loads per lane in flight in phases B and C
 
 struct ResArgs {
   SpmmArgs s;
@@ -573,11 +582,17 @@ __device__ __forceinline__ float4 ldcg_f4(const float* p) {
   return __ldcg(reinterpret_cast<const float4*>(p));
 }
 
-// wait until the generation counter moves past `g` (bounded; sets flags[3] on timeout)
-__device__ __forceinline__ void wait_generation(unsigned* gen, unsigned g, int* flags) {
+// count this block in at the next synchronisation; the __syncthreads before thread 0's release
+// orders the whole block's writes (and its reads of earlier partials) before it
+__device__ __forceinline__ void res_arrive(unsigned* arr) {
+  __syncthreads();
+  if (threadIdx.x == 0) red_release_add(arr, 1u);
+}
+// bounded wait until `target` arrivals (sets flags[3] on timeout)
+__device__ __forceinline__ void res_wait(const unsigned* arr, unsigned target, int* flags) {
   if (threadIdx.x == 0) {
     unsigned spins = 0;
-    while (ld_acquire(gen) == g) {  // one L2 round trip per poll: ~2^22 polls is seconds
+    while ((int)(ld_acquire(arr) - target) < 0) {  // one L2 round trip per poll: ~2^22 is seconds
       if (++spins > (1u << 22)) {
         atomicOr(&flags[3], 1);
         break;
@@ -587,31 +602,17 @@ __device__ __forceinline__ void wait_generation(unsigned* gen, unsigned g, int* 
   __syncthreads();
 }
 
-// plain grid barrier on (count, generation); every block calls it the same number of times.
-// The __syncthreads before thread 0's acquire-release arrival orders the whole block's writes.
-__device__ __forceinline__ void grid_barrier(unsigned* cnt, unsigned* gen, int* flags) {
-  __shared__ unsigned s_g;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    s_g = ld_acquire(gen);
-    if (atom_add_acq_rel(cnt, 1u) == gridDim.x - 1) {
-      atomicExch(cnt, 0u);
-      red_release_add(gen, 1u);
-    }
-  }
-  __syncthreads();
-  wait_generation(gen, s_g, flags);
-}
-
 template <int LPR, int VPL, bool WEIGHTED>
 __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   extern __shared__ __align__(16) float dsm[];
   const SpmmArgs& a = ra.s;
   const VecArgs& va = ra.v;
   constexpr int GPB = PT / LPR;
+  constexpr int NU = RU > VPL ? RU / VPL : 1;  // rows whose loads are in flight together
   const int gl = threadIdx.x & (LPR - 1);
   const int gi = threadIdx.x / LPR;
   const int ld = a.ld, nvec = ld >> 2;
+  const int G = gridDim.x;
   const unsigned gm = group_mask<LPR>();
   const int64_t r0 = (int64_t)blockIdx.x * ra.rb;
   const int nrows = (int)max((int64_t)0, min((int64_t)a.n, r0 + ra.rb) - r0);
@@ -619,14 +620,31 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   float* aps = rs + (size_t)ra.rb * ld;                // [rb][ld]  Ap of own rows
   float* comb = aps + (size_t)ra.rb * ld;              // [GPB][ld] heavy-row slices
   float2* sbuf = reinterpret_cast<float2*>(comb + (size_t)GPB * ld);  // [ld]
-  float2* scratch = sbuf + ld;                         // [PWARPS][PCH]
-  __shared__ unsigned s_gen;
+  float2* scratch = sbuf + ld;                         // [PWARPS][PCH] = 2 * PT entries
+  float2* part_pap = a.cr.part1;                       // [G][ld] block partials of p.Ap
+  float2* part_rr = a.cr.part1 + (size_t)G * ld;       // [G][ld] block partials of r.r
+  unsigned* arrivals = va.gen;
+  // per-column CG state, the same in every block
+  __shared__ double s_rr[RMAXLD], s_yy[RMAXLD];
+  __shared__ __align__(16) float s_alpha[RMAXLD], s_beta[RMAXLD];
+  __shared__ __align__(16) int s_active[RMAXLD];
+  __shared__ int s_iters[RMAXLD], s_conv[RMAXLD];
   __shared__ int64_t s_h0, s_h1;
-  unsigned* bar_cnt = va.gen + 1;
 
   for (int idx = threadIdx.x; idx < nrows * nvec; idx += PT) {
     const int i = idx / nvec, q = idx % nvec;
     reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = ldcg_f4(va.R + (size_t)(r0 + i) * ld + 4 * q);
+  }
+  int any = 0;
+  for (int c = threadIdx.x; c < ld; c += PT) {
+    s_rr[c] = __ldcg(va.rr + c);
+    s_yy[c] = __ldcg(va.yy + c);
+    s_alpha[c] = 0.f;
+    s_beta[c] = 0.f;
+    s_active[c] = __ldcg(va.active + c);
+    s_iters[c] = __ldcg(va.iters + c);
+    s_conv[c] = __ldcg(va.conv + c);
+    any |= s_active[c];
   }
   if (threadIdx.x == 0) {  // this block's slice of the ascending heavy-row list
     const int64_t nh = a.nheavy ? *a.nheavy : 0;
@@ -643,18 +661,20 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     }
     s_h1 = lo;
   }
-  __syncthreads();
+  any = __syncthreads_or(any);
 
-  while (true) {
-    if (*(volatile int*)&va.flags[0] == 0 || *(volatile int*)&va.flags[3] != 0) break;
+  unsigned nsync = 0;
+  float2 dot[VPL][4];
+  while (any) {
+    if (*(volatile int*)&va.flags[3] != 0) break;
     // ---------------- A: Ap = L_eps p on own rows, p.Ap
-    float2 dot[VPL][4];
+    if (nsync) res_wait(arrivals, nsync * G, va.flags);  // every block's p is written
 #pragma unroll
     for (int v = 0; v < VPL; ++v)
 #pragma unroll
       for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
-    for (int64_t h = s_h0; h < s_h1; ++h) {
-      const int64_t u = a.heavy[h];
+    for (int64_t hh = s_h0; hh < s_h1; ++hh) {
+      const int64_t u = a.heavy[hh];
       const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
       const int64_t per = (j1 - j0 + GPB - 1) / GPB;
       const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
@@ -665,7 +685,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
         acc[v] = f4_zero();
       }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, nvec, pu, s0, s1, acc);
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, s0, s1, acc);
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
@@ -710,7 +730,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
         acc[v] = f4_zero();
       }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, nvec, pu, j0, j1, acc);
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, j0, j1, acc);
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
@@ -727,28 +747,24 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
       }
     }
-    if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
-    __syncthreads();
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    if (grid_colreduce_flat(a.cr, sbuf, sbuf, scratch, ld)) {
-      for (int c = threadIdx.x; c < ld; c += PT) {
-        const double v = df_value(sbuf[c]);
-        float al = 0.f;
-        if (*(volatile int*)&va.active[c]) {
-          const double q = *(volatile double*)&va.rr[c] / v;
-          if (!(v > 0.0) || !isfinite(q)) {
-            va.active[c] = 0;
-            atomicOr(&va.flags[1], 1);
-          } else {
-            al = (float)q;
-          }
+    for (int c = threadIdx.x; c < ld; c += PT) part_pap[(size_t)blockIdx.x * ld + c] = sbuf[c];
+    res_arrive(arrivals);
+    res_wait(arrivals, ++nsync * G, va.flags);
+    colsum_rows(part_pap, G, ld, sbuf, scratch);
+    for (int c = threadIdx.x; c < ld; c += PT) {
+      const double v = df_value(sbuf[c]);
+      float al = 0.f;
+      if (s_active[c]) {
+        const double q = s_rr[c] / v;
+        if (!(v > 0.0) || !isfinite(q)) {
+          s_active[c] = 0;
+          if (blockIdx.x == 0) atomicOr(&va.flags[1], 1);
+        } else {
+          al = (float)q;
         }
-        va.alpha[c] = al;
       }
-      __syncthreads();
-      if (threadIdx.x == 0) red_release_add(va.gen, 1u);  // orders the block's writes above
-    } else {
-      wait_generation(va.gen, s_gen, va.flags);
+      s_alpha[c] = al;
     }
     __syncthreads();
 
@@ -757,98 +773,648 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
-      al[v] = q < nvec ? ldcg_f4(va.alpha + 4 * q) : f4_zero();
-    }
-#pragma unroll
-    for (int v = 0; v < VPL; ++v)
-#pragma unroll
+      al[v] = q < nvec ? reinterpret_cast<const float4*>(s_alpha)[q] : f4_zero();
       for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
-    for (int i = gi; i < nrows; i += GPB) {
-      const size_t ig = (size_t)(r0 + i) * ld;
+    }
+    for (int i0 = gi; i0 < nrows; i0 += NU * GPB) {
+      float4 p[NU][VPL], x[NU][VPL];
 #pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        if (q >= nvec) continue;
-        const float4 p = ldcg_f4(a.P + ig + 4 * q);
-        float4 x = *reinterpret_cast<const float4*>(va.X + ig + 4 * q);
-        float4 r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
-        const float4 ap = reinterpret_cast<const float4*>(aps + (size_t)i * ld)[q];
-        x.x = fmaf(al[v].x, p.x, x.x);
-        x.y = fmaf(al[v].y, p.y, x.y);
-        x.z = fmaf(al[v].z, p.z, x.z);
-        x.w = fmaf(al[v].w, p.w, x.w);
-        r.x = fmaf(-al[v].x, ap.x, r.x);
-        r.y = fmaf(-al[v].y, ap.y, r.y);
-        r.z = fmaf(-al[v].z, ap.z, r.z);
-        r.w = fmaf(-al[v].w, ap.w, r.w);
-        *reinterpret_cast<float4*>(va.X + ig + 4 * q) = x;
-        reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = r;
-        dot[v][0] = df_fma(dot[v][0], r.x, r.x);
-        dot[v][1] = df_fma(dot[v][1], r.y, r.y);
-        dot[v][2] = df_fma(dot[v][2], r.z, r.z);
-        dot[v][3] = df_fma(dot[v][3], r.w, r.w);
-      }
-    }
-    if (threadIdx.x == 0) s_gen = ld_acquire(va.gen);
-    __syncthreads();
-    block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    if (grid_colreduce_flat(a.cr, sbuf, sbuf, scratch, ld)) {
-      int any = 0;
-      for (int c = threadIdx.x; c < ld; c += PT) {
-        float be = 0.f;
-        int act = *(volatile int*)&va.active[c];
-        if (act) {
-          const double rn = df_value(sbuf[c]);
-          const int it = *(volatile int*)&va.iters[c] + 1;
-          va.iters[c] = it;
-          if (!isfinite(rn)) {
-            act = 0;
-            atomicOr(&va.flags[1], 1);
-          } else {
-            be = (float)(rn / *(volatile double*)&va.rr[c]);
-            va.rr[c] = rn;
-            if (rn <= va.tol2 * *(volatile double*)&va.yy[c]) {
-              va.conv[c] = 1;
-              act = 0;
-            } else if (it >= va.max_iter) {
-              act = 0;
-            }
+      for (int k = 0; k < NU; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int i = i0 + k * GPB, q = gl + LPR * v;
+          if (i < nrows && q < nvec) {
+            const size_t o = (size_t)(r0 + i) * ld + 4 * q;
+            p[k][v] = ldcg_f4(a.P + o);
+            x[k][v] = *reinterpret_cast<const float4*>(va.X + o);
           }
-          va.active[c] = act;
         }
-        va.beta[c] = be;
-        any |= act;
-      }
-      any = __syncthreads_or(any);
-      if (threadIdx.x == 0) {
-        va.flags[0] = any;
-        red_release_add(va.gen, 1u);  // orders the block's writes above
-      }
-    } else {
-      wait_generation(va.gen, s_gen, va.flags);
+#pragma unroll
+      for (int k = 0; k < NU; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int i = i0 + k * GPB, q = gl + LPR * v;
+          if (i >= nrows || q >= nvec) continue;
+          float4 xx = x[k][v], r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
+          const float4 pp = p[k][v], ap = reinterpret_cast<const float4*>(aps + (size_t)i * ld)[q];
+          xx.x = fmaf(al[v].x, pp.x, xx.x);
+          xx.y = fmaf(al[v].y, pp.y, xx.y);
+          xx.z = fmaf(al[v].z, pp.z, xx.z);
+          xx.w = fmaf(al[v].w, pp.w, xx.w);
+          r.x = fmaf(-al[v].x, ap.x, r.x);
+          r.y = fmaf(-al[v].y, ap.y, r.y);
+          r.z = fmaf(-al[v].z, ap.z, r.z);
+          r.w = fmaf(-al[v].w, ap.w, r.w);
+          *reinterpret_cast<float4*>(va.X + (size_t)(r0 + i) * ld + 4 * q) = xx;
+          reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = r;
+          dot[v][0] = df_fma(dot[v][0], r.x, r.x);
+          dot[v][1] = df_fma(dot[v][1], r.y, r.y);
+          dot[v][2] = df_fma(dot[v][2], r.z, r.z);
+          dot[v][3] = df_fma(dot[v][3], r.w, r.w);
+        }
     }
-    __syncthreads();
+    block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
+    for (int c = threadIdx.x; c < ld; c += PT) part_rr[(size_t)blockIdx.x * ld + c] = sbuf[c];
+    res_arrive(arrivals);
+    res_wait(arrivals, ++nsync * G, va.flags);
+    colsum_rows(part_rr, G, ld, sbuf, scratch);
+    any = 0;
+    for (int c = threadIdx.x; c < ld; c += PT) {
+      float be = 0.f;
+      int act = s_active[c];
+      if (act) {
+        const double rn = df_value(sbuf[c]);
+        const int it = s_iters[c] + 1;
+        s_iters[c] = it;
+        if (!isfinite(rn)) {
+          act = 0;
+          if (blockIdx.x == 0) atomicOr(&va.flags[1], 1);
+        } else {
+          be = (float)(rn / s_rr[c]);
+          s_rr[c] = rn;
+          if (rn <= va.tol2 * s_yy[c]) {
+            s_conv[c] = 1;
+            act = 0;
+          } else if (it >= va.max_iter) {
+            act = 0;
+          }
+        }
+        s_active[c] = act;
+      }
+      s_beta[c] = be;
+      any |= act;
+    }
+    any = __syncthreads_or(any);  // the same in every block
+    if (!any) break;
 
     // ---------------- C: p = r + beta p on active columns
+    int4 act[VPL];
+    float4 be[VPL];
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
-      if (q >= nvec) continue;
-      const int4 act = __ldcg(reinterpret_cast<const int4*>(va.active + 4 * q));
-      if (!(act.x | act.y | act.z | act.w)) continue;
-      const float4 be = ldcg_f4(va.beta + 4 * q);
-      for (int i = gi; i < nrows; i += GPB) {
-        const size_t ig = (size_t)(r0 + i) * ld + 4 * q;
-        const float4 r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
-        float4 p = ldcg_f4(a.P + ig);
-        if (act.x) p.x = fmaf(be.x, p.x, r.x);
-        if (act.y) p.y = fmaf(be.y, p.y, r.y);
-        if (act.z) p.z = fmaf(be.z, p.z, r.z);
-        if (act.w) p.w = fmaf(be.w, p.w, r.w);
-        *reinterpret_cast<float4*>(const_cast<float*>(a.P) + ig) = p;
+      act[v] = q < nvec ? reinterpret_cast<const int4*>(s_active)[q] : make_int4(0, 0, 0, 0);
+      be[v] = q < nvec ? reinterpret_cast<const float4*>(s_beta)[q] : f4_zero();
+    }
+    for (int i0 = gi; i0 < nrows; i0 += NU * GPB) {
+      float4 p[NU][VPL];
+#pragma unroll
+      for (int k = 0; k < NU; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int i = i0 + k * GPB, q = gl + LPR * v;
+          if (i < nrows && (act[v].x | act[v].y | act[v].z | act[v].w))
+            p[k][v] = ldcg_f4(a.P + (size_t)(r0 + i) * ld + 4 * q);
+        }
+#pragma unroll
+      for (int k = 0; k < NU; ++k)
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          const int i = i0 + k * GPB, q = gl + LPR * v;
+          if (i >= nrows || !(act[v].x | act[v].y | act[v].z | act[v].w)) continue;
+          const float4 r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
+          float4 pp = p[k][v];
+          if (act[v].x) pp.x = fmaf(be[v].x, pp.x, r.x);
+          if (act[v].y) pp.y = fmaf(be[v].y, pp.y, r.y);
+          if (act[v].z) pp.z = fmaf(be[v].z, pp.z, r.z);
+          if (act[v].w) pp.w = fmaf(be[v].w, pp.w, r.w);
+          *reinterpret_cast<float4*>(const_cast<float*>(a.P) + (size_t)(r0 + i) * ld + 4 * q) = pp;
+        }
+    }
+    res_arrive(arrivals);
+    ++nsync;
+  }
+  // the per-column results, identical in every block
+  if (blockIdx.x == 0)
+    for (int c = threadIdx.x; c < ld; c += PT) {
+      va.rr[c] = s_rr[c];
+      va.iters[c] = s_iters[c];
+      va.conv[c] = s_conv[c];
+      va.active[c] = s_active[c];
+    }
+}
+
+// ---------------------------------------------------------------------------- cluster CG
+// The kc columns of Eq. 5 are independent systems, so the solve can also be split by columns:
+// a thread-block cluster of CS blocks owns a group of 16 columns for every row and runs the whole
+// solve of its group; clusters never wait on one another.  Block k of a cluster owns the rows
+// [b_k, b_k+1) (equal shares of the neighbour lists, at most rbmax rows): their r and Ap live in
+// its shared memory, x and p in global memory (p is gathered by the cluster's other blocks, from
+// L2).  Four lanes take one light row, a float4 of the group's columns each, so a neighbour costs
+// one 64-byte line; the next row's bounds and column indices are fetched while the current row's
+// neighbours are in flight.  Rows heavier than H are split over the whole block.  Per-column dot
+// products are combined in a fixed order: within a block by warp shuffles and shared memory,
+// across the cluster by every block reading every block's partial through distributed shared
+// memory, so all blocks of a cluster derive the same alpha, beta and stop decisions.
+// Per iteration: A (Ap, p.Ap) | B (x, r, r.r) | C (p), each closed by a hardware cluster barrier.
+constexpr int CT = 384;
+constexpr int CWARPS = CT / 32;
+constexpr int CL = 4;            // lanes per row
+constexpr int CGR = CT / CL;     // rows in flight per block
+constexpr int CW = 4 * CL;       // columns per group
+constexpr int CHMAX = 256;       // heavy rows per block
+constexpr int CMAXS = 16;        // largest cluster
+constexpr int CU = 16;           // neighbour rows per batch
+constexpr int CIDX = CU / CL;    // column indices each lane fetches per batch
+constexpr int CUNROLL = 4;       // rows per lane in flight in the vector phases
+
+struct ClusterArgs {
+  const int64_t* row_ptr;
+  const int32_t* col;
+  const float* val;
+  int32_t n, ld, kc;
+  float eps;
+  double tol2;
+  int32_t max_iter;
+  int32_t rbmax;  // rows of r and Ap a block's shared memory holds
+  const float* Y;
+  float* X;
+  float* P;
+  double *yy, *rr;
+  int *iters, *conv, *flags;
+};
+
+__device__ __forceinline__ unsigned cluster_rank() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ unsigned cluster_size() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ unsigned cluster_index() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+// every thread of every block of the cluster; orders shared and global memory at cluster scope
+__device__ __forceinline__ void cluster_barrier() {
+  asm volatile(
+      "barrier.cluster.arrive.release.aligned;\n\t"
+      "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// float2 at the same shared-memory offset in block `rank` of this cluster
+__device__ __forceinline__ float2 ld_cluster_f2(const float2* local, unsigned rank) {
+  const unsigned a = (unsigned)__cvta_generic_to_shared(local);
+  unsigned ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+  float2 v;
+  asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(ra) : "memory");
+  return v;
+}
+
+struct ClusterShared {
+  float2 red[2][CW];  // this block's partials (two slots: consecutive reductions)
+  float2 wsum[CWARPS][CW];
+  float2 tot[CW];
+  float4 comb[CWARPS][CL];
+  double rr[CW], yy[CW];
+  float alpha[CW], beta[CW];
+  int active[CW], iters[CW], conv[CW];
+  int64_t samp[CT];
+  int32_t b[CMAXS + 1];
+  int32_t heavy[CHMAX];
+  int wcnt[CWARPS];
+  int nheavy;
+};
+
+// d (per-lane partials of its 4 columns) -> cl.tot: block sum in warp/lane order, then the
+// cluster's block partials in rank order; every block of the cluster obtains the same totals
+__device__ __forceinline__ void cluster_colsum(float2 (&d)[4], ClusterShared& cl, int slot, int S) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = CL; off < 32; off <<= 1)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      float2 o;
+      o.x = __shfl_xor_sync(0xffffffffu, d[t].x, off);
+      o.y = __shfl_xor_sync(0xffffffffu, d[t].y, off);
+      d[t] = df_add(d[t], o);
+    }
+  if (lane < CL)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) cl.wsum[warp][4 * lane + t] = d[t];
+  __syncthreads();
+  if (threadIdx.x < CW) {
+    float2 acc = make_float2(0.f, 0.f);
+    for (int w = 0; w < CWARPS; ++w) acc = df_add(acc, cl.wsum[w][threadIdx.x]);
+    cl.red[slot][threadIdx.x] = acc;
+  }
+  cluster_barrier();
+  if (threadIdx.x < CW) {
+    float2 v[CMAXS];
+#pragma unroll
+    for (int k = 0; k < CMAXS; ++k)
+      v[k] = k < S ? ld_cluster_f2(&cl.red[slot][threadIdx.x], k) : make_float2(0.f, 0.f);
+    float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < CMAXS; ++k)
+      if (k < S) acc = df_add(acc, v[k]);
+    cl.tot[threadIdx.x] = acc;
+  }
+  __syncthreads();
+}
+
+// column indices (and weights) of neighbours [jb, jb + CU) within [jb, j1): lane gl holds
+// entries jb + gl + CL * t
+template <bool WEIGHTED>
+__device__ __forceinline__ void cluster_fetch_idx(const ClusterArgs& a, int gl, int64_t jb,
+                                                  int64_t j1, int (&c)[CIDX], float (&w)[CIDX]) {
+#pragma unroll
+  for (int t = 0; t < CIDX; ++t) {
+    const int64_t j = jb + gl + CL * t;
+    c[t] = j < j1 ? __ldg(a.col + j) : 0;
+    w[t] = j < j1 ? (WEIGHTED ? __ldg(a.val + j) : 1.f) : 0.f;
+  }
+}
+
+// acc += sum over the batch [jb, min(jb + CU, j1)) of w_j (p_u - p_{col_j}) for this lane's
+// float4.  Slots past j1 load p_u itself, so they add exactly zero.
+template <bool WEIGHTED>
+__device__ __forceinline__ void cluster_batch(const ClusterArgs& a, bool valid, size_t qoff,
+                                              float4 pu, const int (&c)[CIDX],
+                                              const float (&w)[CIDX], int64_t jb, int64_t j1,
+                                              unsigned gm, float4& acc) {
+  float4 v[CU];
+#pragma unroll
+  for (int k = 0; k < CU; ++k) {
+    // entry jb + k sits in lane k % CL, slot k / CL
+    const int ck = __shfl_sync(gm, c[k / CL], k % CL, CL);
+    v[k] = valid && jb + k < j1
+               ? __ldcg(reinterpret_cast<const float4*>(a.P + (size_t)ck * a.ld + qoff))
+               : pu;
+  }
+#pragma unroll
+  for (int k = 0; k < CU; ++k) {
+    if (WEIGHTED) {
+      const float wk = __shfl_sync(gm, w[k / CL], k % CL, CL);
+      acc.x = fmaf(wk, pu.x - v[k].x, acc.x);
+      acc.y = fmaf(wk, pu.y - v[k].y, acc.y);
+      acc.z = fmaf(wk, pu.z - v[k].z, acc.z);
+      acc.w = fmaf(wk, pu.w - v[k].w, acc.w);
+    } else {
+      acc.x += pu.x - v[k].x;
+      acc.y += pu.y - v[k].y;
+      acc.z += pu.z - v[k].z;
+      acc.w += pu.w - v[k].w;
+    }
+  }
+}
+
+__device__ __forceinline__ void dot4(float2 (&d)[4], float4 a, float4 b) {
+  d[0] = df_fma(d[0], a.x, b.x);
+  d[1] = df_fma(d[1], a.y, b.y);
+  d[2] = df_fma(d[2], a.z, b.z);
+  d[3] = df_fma(d[3], a.w, b.w);
+}
+__device__ __forceinline__ float4 fma4(float4 s, float4 a, float4 b) {  // s * a + b
+  return make_float4(fmaf(s.x, a.x, b.x), fmaf(s.y, a.y, b.y), fmaf(s.z, a.z, b.z),
+                     fmaf(s.w, a.w, b.w));
+}
+__device__ __forceinline__ float4 eps_fma4(float e, float4 p, float4 acc) {
+  return make_float4(fmaf(e, p.x, acc.x), fmaf(e, p.y, acc.y), fmaf(e, p.z, acc.z),
+                     fmaf(e, p.w, acc.w));
+}
+
+template <bool WEIGHTED>
+__global__ void __launch_bounds__(CT, 1) k_cg_cluster(ClusterArgs a) {
+  extern __shared__ __align__(16) float4 csm[];
+  __shared__ ClusterShared cl;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int gl = tid & (CL - 1), gi = tid / CL;
+  const unsigned gm = 0xfu << (lane & ~(CL - 1));
+  const int S = (int)cluster_size(), rank = (int)cluster_rank();
+  const int q = CL * (int)cluster_index() + gl;  // this lane's float4 slot of the row
+  const bool valid = q < (a.ld >> 2);
+  const size_t qoff = 4 * (size_t)q;
+  const int rbmax = a.rbmax;
+  float4* rs = csm;                 // [rbmax][CL] r of own rows
+  float4* aps = csm + CL * rbmax;   // [rbmax][CL] Ap of own rows
+
+  // ---- row split: S equal shares of the neighbour lists, each of at most rbmax rows
+  const int64_t nnz = a.row_ptr[a.n];
+  cl.samp[tid] = a.row_ptr[(int64_t)tid * a.n / (CT - 1)];
+  __syncthreads();
+  if (tid <= S) {
+    const int64_t target = (int64_t)tid * nnz / S;
+    int f = 0, fh = CT - 1;  // first sample f with samp[f] >= target (samp[CT - 1] = nnz)
+    while (f < fh) {
+      const int mid = (f + fh) >> 1;
+      if (cl.samp[mid] < target) f = mid + 1; else fh = mid;
+    }
+    int64_t lo = f > 0 ? (int64_t)(f - 1) * a.n / (CT - 1) : 0;
+    int64_t hi = (int64_t)f * a.n / (CT - 1);
+    while (lo < hi) {  // first row u with row_ptr[u] >= target
+      const int64_t mid = (lo + hi) >> 1;
+      if (a.row_ptr[mid] < target) lo = mid + 1; else hi = mid;
+    }
+    cl.b[tid] = (int32_t)lo;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int32_t b = 0;
+    cl.b[0] = 0;
+    for (int k = 0; k < S; ++k) {
+      const int64_t need = (int64_t)a.n - (int64_t)(S - k - 1) * rbmax;
+      int64_t nb = cl.b[k + 1];
+      nb = max(nb, max((int64_t)b, need));
+      nb = min(nb, (int64_t)b + rbmax);
+      b = (int32_t)nb;
+      cl.b[k + 1] = b;
+    }
+    int ok = b == a.n;
+    for (int k = 0; k < S; ++k) ok &= cl.b[k + 1] - cl.b[k] <= rbmax;
+    cl.nheavy = ok;  // reused below; the host sizes rbmax so that this holds
+  }
+  __syncthreads();
+  if (!cl.nheavy) {  // the same outcome in every block: none reaches a cluster barrier
+    if (tid == 0 && rank == 0) atomicOr(&a.flags[1], 1);
+    return;
+  }
+  __syncthreads();
+  const int32_t b0 = cl.b[rank];
+  const int nr = cl.b[rank + 1] - b0;
+  const int64_t* rp = a.row_ptr + b0;
+  const int64_t nnz_b = rp[nr] - rp[0];
+  const int64_t H = max((int64_t)64, (nnz_b + CHMAX - 1) / CHMAX);  // at most CHMAX heavy rows
+
+  // ---- heavy rows of this block, ascending
+  if (tid == 0) cl.nheavy = 0;
+  __syncthreads();
+  for (int base = 0; base < nr; base += CT) {
+    const int i = base + tid;
+    const bool hv = i < nr && rp[i + 1] - rp[i] > H;
+    const unsigned bal = __ballot_sync(0xffffffffu, hv);
+    if (lane == 0) cl.wcnt[warp] = __popc(bal);
+    __syncthreads();
+    int off = cl.nheavy, tot = 0;
+    for (int w = 0; w < CWARPS; ++w) {
+      if (w < warp) off += cl.wcnt[w];
+      tot += cl.wcnt[w];
+    }
+    if (hv) cl.heavy[off + __popc(bal & ((1u << lane) - 1u))] = i;
+    __syncthreads();
+    if (tid == 0) cl.nheavy += tot;
+    __syncthreads();
+  }
+  const int nheavy = cl.nheavy;
+
+  // ---- r = p = y (columns beyond kc zero), x = 0, y.y
+  float2 d[4];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) d[t] = make_float2(0.f, 0.f);
+  for (int i = gi; i < nr; i += CGR) {
+    const size_t o = (size_t)(b0 + i) * a.ld + qoff;
+    float4 y = f4_zero();
+    if (valid) {
+      y = ld_f4(a.Y + o);
+      const int cb = 4 * q;
+      if (cb + 0 >= a.kc) y.x = 0.f;
+      if (cb + 1 >= a.kc) y.y = 0.f;
+      if (cb + 2 >= a.kc) y.z = 0.f;
+      if (cb + 3 >= a.kc) y.w = 0.f;
+      *reinterpret_cast<float4*>(a.P + o) = y;
+      *reinterpret_cast<float4*>(a.X + o) = f4_zero();
+    }
+    rs[i * CL + gl] = y;
+    dot4(d, y, y);
+  }
+  cluster_colsum(d, cl, 0, S);  // its barrier also publishes p to the cluster
+  if (tid < CW) {
+    const int c = 4 * CL * (int)cluster_index() + tid;
+    const double v = df_value(cl.tot[tid]);
+    int act = 0, cv = 1;
+    if (c < a.kc) {
+      if (!isfinite(v)) {
+        if (rank == 0) atomicOr(&a.flags[1], 1);
+        cv = 0;
+      } else if (v > 0.0 && !(v <= a.tol2 * v)) {
+        act = 1;
+        cv = 0;
       }
     }
-    grid_barrier(bar_cnt, va.gen, va.flags);
+    cl.yy[tid] = v;
+    cl.rr[tid] = v;
+    cl.iters[tid] = 0;
+    cl.active[tid] = act;
+    cl.conv[tid] = cv;
+  }
+  int any = __syncthreads_or(tid < CW && cl.active[tid]);
+
+  int slot = 1;
+  while (any) {
+    // ---------------- A: Ap = L_eps p on own rows, p.Ap
+#pragma unroll
+    for (int t = 0; t < 4; ++t) d[t] = make_float2(0.f, 0.f);
+    {
+      // light rows, software-pipelined: row i's first batch of indices and row i + CGR's bounds
+      // are in registers when row i starts; row i + CGR's first indices are fetched with it
+      int i = gi;
+      int64_t j0 = 0, j1 = 0, nj0 = 0, nj1 = 0;
+      if (i < nr) {
+        j0 = rp[i];
+        j1 = rp[i + 1];
+      }
+      if (i + CGR < nr) {
+        nj0 = rp[i + CGR];
+        nj1 = rp[i + CGR + 1];
+      }
+      bool hv = j1 - j0 > H;
+      int c[CIDX], cn[CIDX];
+      float w[CIDX], wn[CIDX];
+      cluster_fetch_idx<WEIGHTED>(a, gl, j0, hv ? j0 : j1, c, w);
+      for (; i < nr; i += CGR) {
+        const bool nhv = nj1 - nj0 > H;
+        cluster_fetch_idx<WEIGHTED>(a, gl, nj0, nhv ? nj0 : nj1, cn, wn);
+        int64_t nnj0 = 0, nnj1 = 0;
+        if (i + 2 * CGR < nr) {
+          nnj0 = rp[i + 2 * CGR];
+          nnj1 = rp[i + 2 * CGR + 1];
+        }
+        if (!hv) {
+          const float4 pu = valid ? __ldcg(reinterpret_cast<const float4*>(
+                                        a.P + (size_t)(b0 + i) * a.ld + qoff))
+                                  : f4_zero();
+          float4 acc = f4_zero();
+          cluster_batch<WEIGHTED>(a, valid, qoff, pu, c, w, j0, j1, gm, acc);
+          for (int64_t jb = j0 + CU; jb < j1; jb += CU) {  // rows longer than one batch
+            cluster_fetch_idx<WEIGHTED>(a, gl, jb, j1, c, w);
+            cluster_batch<WEIGHTED>(a, valid, qoff, pu, c, w, jb, j1, gm, acc);
+          }
+          const float4 o = eps_fma4(a.eps, pu, acc);
+          aps[i * CL + gl] = o;
+          dot4(d, pu, o);
+        }
+        j0 = nj0;
+        j1 = nj1;
+        hv = nhv;
+        nj0 = nnj0;
+        nj1 = nnj1;
+#pragma unroll
+        for (int t = 0; t < CIDX; ++t) {
+          c[t] = cn[t];
+          w[t] = wn[t];
+        }
+      }
+    }
+    for (int h = 0; h < nheavy; ++h) {  // the whole block on one row, slices combined in order
+      const int i = cl.heavy[h];
+      const int64_t j0 = rp[i], j1 = rp[i + 1];
+      const int64_t per = (j1 - j0 + CGR - 1) / CGR;
+      const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
+      const float4 pu = valid ? __ldcg(reinterpret_cast<const float4*>(
+                                    a.P + (size_t)(b0 + i) * a.ld + qoff))
+                              : f4_zero();
+      float4 acc = f4_zero();
+      int c[CIDX];
+      float w[CIDX];
+      for (int64_t jb = s0; jb < s1; jb += CU) {
+        cluster_fetch_idx<WEIGHTED>(a, gl, jb, s1, c, w);
+        cluster_batch<WEIGHTED>(a, valid, qoff, pu, c, w, jb, s1, gm, acc);
+      }
+#pragma unroll
+      for (int off = CL; off < 32; off <<= 1) {
+        acc.x += __shfl_xor_sync(0xffffffffu, acc.x, off);
+        acc.y += __shfl_xor_sync(0xffffffffu, acc.y, off);
+        acc.z += __shfl_xor_sync(0xffffffffu, acc.z, off);
+        acc.w += __shfl_xor_sync(0xffffffffu, acc.w, off);
+      }
+      if (lane < CL) cl.comb[warp][lane] = acc;
+      __syncthreads();
+      if (tid < CL) {
+        float4 s = f4_zero();
+        for (int wp = 0; wp < CWARPS; ++wp) {
+          const float4 cv = cl.comb[wp][tid];
+          s = make_float4(s.x + cv.x, s.y + cv.y, s.z + cv.z, s.w + cv.w);
+        }
+        const float4 o = eps_fma4(a.eps, pu, s);
+        aps[i * CL + tid] = o;
+        dot4(d, pu, o);
+      }
+      __syncthreads();
+    }
+    cluster_colsum(d, cl, slot, S);
+    slot ^= 1;
+    if (tid < CW) {
+      float al = 0.f;
+      if (cl.active[tid]) {
+        const double v = df_value(cl.tot[tid]);
+        const double qq = cl.rr[tid] / v;
+        if (!(v > 0.0) || !isfinite(qq)) {
+          cl.active[tid] = 0;
+          if (rank == 0) atomicOr(&a.flags[1], 1);
+        } else {
+          al = (float)qq;
+        }
+      }
+      cl.alpha[tid] = al;
+    }
+    __syncthreads();
+
+    // ---------------- B: x += alpha p, r -= alpha Ap, r.r
+    {
+      const float4 al = make_float4(cl.alpha[4 * gl], cl.alpha[4 * gl + 1], cl.alpha[4 * gl + 2],
+                                    cl.alpha[4 * gl + 3]);
+      const float4 nal = make_float4(-al.x, -al.y, -al.z, -al.w);
+#pragma unroll
+      for (int t = 0; t < 4; ++t) d[t] = make_float2(0.f, 0.f);
+      if (valid) {
+        for (int i0 = gi; i0 < nr; i0 += CUNROLL * CGR) {
+          float4 p[CUNROLL], x[CUNROLL];
+#pragma unroll
+          for (int k = 0; k < CUNROLL; ++k) {
+            const int i = i0 + k * CGR;
+            if (i < nr) {
+              const size_t o = (size_t)(b0 + i) * a.ld + qoff;
+              p[k] = __ldcg(reinterpret_cast<const float4*>(a.P + o));
+              x[k] = *reinterpret_cast<const float4*>(a.X + o);
+            }
+          }
+#pragma unroll
+          for (int k = 0; k < CUNROLL; ++k) {
+            const int i = i0 + k * CGR;
+            if (i < nr) {
+              const size_t o = (size_t)(b0 + i) * a.ld + qoff;
+              *reinterpret_cast<float4*>(a.X + o) = fma4(al, p[k], x[k]);
+              const float4 r = fma4(nal, aps[i * CL + gl], rs[i * CL + gl]);
+              rs[i * CL + gl] = r;
+              dot4(d, r, r);
+            }
+          }
+        }
+      }
+    }
+    cluster_colsum(d, cl, slot, S);
+    slot ^= 1;
+    if (tid < CW) {
+      float be = 0.f;
+      int act = cl.active[tid];
+      if (act) {
+        const double rn = df_value(cl.tot[tid]);
+        const int it = cl.iters[tid] + 1;
+        cl.iters[tid] = it;
+        if (!isfinite(rn)) {
+          act = 0;
+          if (rank == 0) atomicOr(&a.flags[1], 1);
+        } else {
+          be = (float)(rn / cl.rr[tid]);
+          cl.rr[tid] = rn;
+          if (rn <= a.tol2 * cl.yy[tid]) {
+            cl.conv[tid] = 1;
+            act = 0;
+          } else if (it >= a.max_iter) {
+            act = 0;
+          }
+        }
+        cl.active[tid] = act;
+      }
+      cl.beta[tid] = be;
+    }
+    any = __syncthreads_or(tid < CW && cl.active[tid]);
+    if (!any) break;
+
+    // ---------------- C: p = r + beta p on active columns
+    {
+      const int4 act = make_int4(cl.active[4 * gl], cl.active[4 * gl + 1], cl.active[4 * gl + 2],
+                                 cl.active[4 * gl + 3]);
+      const float4 be = make_float4(cl.beta[4 * gl], cl.beta[4 * gl + 1], cl.beta[4 * gl + 2],
+                                    cl.beta[4 * gl + 3]);
+      if (valid && (act.x | act.y | act.z | act.w)) {
+        for (int i0 = gi; i0 < nr; i0 += CUNROLL * CGR) {
+          float4 p[CUNROLL];
+#pragma unroll
+          for (int k = 0; k < CUNROLL; ++k) {
+            const int i = i0 + k * CGR;
+            if (i < nr)
+              p[k] = __ldcg(reinterpret_cast<const float4*>(a.P + (size_t)(b0 + i) * a.ld + qoff));
+          }
+#pragma unroll
+          for (int k = 0; k < CUNROLL; ++k) {
+            const int i = i0 + k * CGR;
+            if (i < nr) {
+              const float4 r = rs[i * CL + gl];
+              if (act.x) p[k].x = fmaf(be.x, p[k].x, r.x);
+              if (act.y) p[k].y = fmaf(be.y, p[k].y, r.y);
+              if (act.z) p[k].z = fmaf(be.z, p[k].z, r.z);
+              if (act.w) p[k].w = fmaf(be.w, p[k].w, r.w);
+              *reinterpret_cast<float4*>(a.P + (size_t)(b0 + i) * a.ld + qoff) = p[k];
+            }
+          }
+        }
+      }
+    }
+    cluster_barrier();
+  }
+  // no block leaves while another may still read its partials
+  cluster_barrier();
+  const int c = 4 * CL * (int)cluster_index() + tid;
+  if (rank == 0 && tid < CW && c < a.ld) {
+    a.yy[c] = cl.yy[tid];
+    a.rr[c] = cl.rr[tid];
+    a.iters[c] = cl.iters[tid];
+    a.conv[c] = cl.conv[tid];
   }
 }
 
@@ -945,6 +1511,8 @@ erc_status launch_update(const VecArgs& va, int grid, cudaStream_t s) {
 }
 
 // ---- resident path selection: the kernel for this shape, its shared memory, and whether it fits
+int resident_lpr(int nvec) { return nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32; }
+
 const void* resident_kernel(int nvec, bool weighted) {
   const void* k = nullptr;
   auto pick = [&](auto lpr, auto vpl) {
@@ -961,21 +1529,23 @@ const void* resident_kernel(int nvec, bool weighted) {
 }
 
 bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const void** kern) {
-  const char* mode = getenv("ERC_CG_MODE");
-  if (mode && strcmp(mode, "graph") == 0) return false;
   const int nvec = ld / 4;
   const void* k = resident_kernel(nvec, g->val != nullptr);
   if (!k) return false;
-  const int lpr = nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32;
+  const int lpr = resident_lpr(nvec);
   const int grid = sm_count();
   const int64_t rows = ((int64_t)g->n + grid - 1) / grid;
   const size_t bytes = 4 * (2 * (size_t)rows * ld + (size_t)(PT / lpr) * ld + 2 * (size_t)ld +
                             2 * (size_t)PWARPS * PCH);
   int dev = 0, optin = 0;
+  cudaFuncAttributes fa;
   if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+      cudaFuncGetAttributes(&fa, k) != cudaSuccess) {
+    cudaGetLastError();
     return false;
-  if (bytes > (size_t)optin) return false;
+  }
+  if (bytes + fa.sharedSizeBytes > (size_t)optin) return false;
   if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) !=
       cudaSuccess) {
     cudaGetLastError();
@@ -1005,6 +1575,95 @@ erc_status launch_resident(const void* kern, const ResArgs& ra, size_t smem, cud
   cfg.numAttrs = 1;
   void* args[] = {const_cast<ResArgs*>(&ra)};
   ERC_CUDA(cudaLaunchKernelExC(&cfg, kern, args));
+  count_launches(1);
+  return ERC_OK;
+}
+
+// ---- cluster path: the largest cluster for which every column group's cluster is resident at
+// once, and shared memory for the rows a block may take
+struct ClusterPlan {
+  const void* k = nullptr;
+  int S = 0, groups = 0;
+  int32_t rbmax = 0;
+  size_t smem = 0;
+};
+
+void cluster_config(const ClusterPlan& pl, cudaStream_t s, cudaLaunchConfig_t* cfg,
+                    cudaLaunchAttribute* attr) {
+  *cfg = cudaLaunchConfig_t{};
+  cfg->gridDim = dim3(pl.groups * pl.S);
+  cfg->blockDim = dim3(CT);
+  cfg->dynamicSmemBytes = pl.smem;
+  cfg->stream = s;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = pl.S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg->attrs = attr;
+  cfg->numAttrs = 1;
+}
+
+bool cluster_plan(const erc_graph* g, int ld, ClusterPlan* pl) {
+  const void* k = g->val ? (const void*)k_cg_cluster<true> : (const void*)k_cg_cluster<false>;
+  int dev = 0, optin = 0;
+  cudaFuncAttributes fa;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+      cudaFuncGetAttributes(&fa, k) != cudaSuccess ||
+      cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  const int64_t row_bytes = 2 * CL * sizeof(float4);  // r and Ap of the group's columns
+  const int64_t cap = ((int64_t)optin - (int64_t)fa.sharedSizeBytes - 1024) / row_bytes;
+  const int groups = (ld / 4 + CL - 1) / CL;
+  for (int S = CMAXS; S >= 1; --S) {
+    const int64_t even = ((int64_t)g->n + S - 1) / S;
+    if (even > cap) break;  // smaller clusters need still more rows per block
+    ClusterPlan p;
+    p.k = k;
+    p.S = S;
+    p.groups = groups;
+    p.rbmax = (int32_t)std::min(cap, even + even / 8 + 32);  // room to balance neighbour lists
+    p.smem = (size_t)p.rbmax * row_bytes;
+    if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      continue;
+    }
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr[1];
+    cluster_config(p, nullptr, &cfg, attr);
+    int nc = 0;
+    if (cudaOccupancyMaxActiveClusters(&nc, k, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      continue;
+    }
+    if (nc < groups) continue;  // one wave: every group's cluster at once
+    *pl = p;
+    return true;
+  }
+  return false;
+}
+
+// Where both single-launch solvers fit, the cheaper per iteration by a model fitted to GB300
+// timings: the resident gather costs ~2.4 ns per 128-byte neighbour line per SM plus ~18 us of
+// synchronisation and vector work; the cluster gather ~2.6 ns per neighbour per block (one
+// request per column group) plus ~10 us.  Small graphs favour the cluster solver.
+bool prefer_cluster(const erc_graph* g, int ld, const ClusterPlan& cp) {
+  const double nnz = 2.0 * (double)g->m;
+  const double lines = std::max(1.0, ld / 32.0);
+  const double t_res = 18.0 + nnz * lines * 2.4e-3 / sm_count();
+  const double t_cl = 10.0 + nnz / cp.S * 2.6e-3;
+  return t_cl < t_res;
+}
+
+erc_status launch_cluster(const ClusterPlan& pl, const ClusterArgs& ca, cudaStream_t s) {
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  cluster_config(pl, s, &cfg, attr);
+  void* args[] = {const_cast<ClusterArgs*>(&ca)};
+  ERC_CUDA(cudaLaunchKernelExC(&cfg, pl.k, args));
   count_launches(1);
   return ERC_OK;
 }
@@ -1200,22 +1859,55 @@ static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y,
   sa.relres_out = relres;
   sa.iters_out = iters;
 
-  k_cg_init<<<grid_for(g->n, vec_threads(nvec) / nvec), vec_threads(nvec), 0, s>>>(va);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-
+  // path: 2 cluster (column groups), 1 resident (one cooperative launch), 0 multi-kernel graph.
+  // ERC_CG_MODE=graph|resident|cluster restricts the choice (testing of every path).
+  const char* mode = getenv("ERC_CG_MODE");
+  ClusterPlan cp;
+  bool cluster = (!mode || strcmp(mode, "cluster") == 0) && cluster_plan(g, ld, &cp);
   int32_t rb = 0;
   size_t smem = 0;
   const void* kres = nullptr;
-  const bool resident = resident_plan(g, ld, &rb, &smem, &kres);
-  if (path) *path = resident ? 1 : 0;
+  bool resident = (!mode || strcmp(mode, "resident") == 0) && resident_plan(g, ld, &rb, &smem, &kres);
+  if (cluster && resident) {
+    if (prefer_cluster(g, ld, cp))
+      resident = false;
+    else
+      cluster = false;
+  }
+  if (path) *path = cluster ? 2 : resident ? 1 : 0;
+  if (!cluster) {  // the cluster kernel initialises its own columns
+    k_cg_init<<<grid_for(g->n, vec_threads(nvec) / nvec), vec_threads(nvec), 0, s>>>(va);
+    count_launches(1);
+    ERC_CUDA(cudaGetLastError());
+  }
   cudaEvent_t ev[2] = {nullptr, nullptr};
   if (solve_us) {
     ERC_CUDA(cudaEventCreate(&ev[0]));
     ERC_CUDA(cudaEventCreate(&ev[1]));
     ERC_CUDA(cudaEventRecord(ev[0], s));
   }
-  if (resident) {
+  if (cluster) {
+    ClusterArgs ca{};
+    ca.row_ptr = g->row_ptr;
+    ca.col = g->col;
+    ca.val = g->val;
+    ca.n = g->n;
+    ca.ld = ld;
+    ca.kc = kc;
+    ca.eps = eps;
+    ca.tol2 = va.tol2;
+    ca.max_iter = max_iter;
+    ca.rbmax = cp.rbmax;
+    ca.Y = Y;
+    ca.X = X;
+    ca.P = w.P;
+    ca.yy = w.yy;
+    ca.rr = w.rr;
+    ca.iters = w.iters;
+    ca.conv = w.conv;
+    ca.flags = w.flags;
+    ERC_TRY(launch_cluster(cp, ca, s));
+  } else if (resident) {
     // the whole solve in one cooperative launch, no host round trips
     ResArgs ra{sa, va, rb};
     ERC_TRY(launch_resident(kres, ra, smem, s));

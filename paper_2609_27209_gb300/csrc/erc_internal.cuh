@@ -184,43 +184,43 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
   return old;
 }
 
-// Single-level variant for grids of a few hundred blocks.  Every block publishes its row, a
-// __syncthreads orders the block's writes before thread 0's acquire-release arrival, and the last
-// block to arrive sums all rows: its threads take fixed segments of the blocks for one column
-// each, then the segments are added in order.  `tmp` is shared scratch of blockDim.x entries.
-// Only cr.cnt[0] is used; the finisher resets it.
-__device__ __forceinline__ bool grid_colreduce_flat(const ColReduce& cr, const float2* bpart,
-                                                    float2* res, float2* tmp, int ld) {
-  __shared__ int s_last;
-  const int G = gridDim.x, b = blockIdx.x;
-  for (int c = threadIdx.x; c < ld; c += blockDim.x) cr.part1[(size_t)b * ld + c] = bpart[c];
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atom_add_acq_rel(&cr.cnt[0], 1u) == (unsigned)(G - 1));
-  __syncthreads();
-  if (!s_last) return false;
+// Ordered column sums of G rows of partials (part: [G][ld] float pairs, written by other blocks
+// of the same launch, read through L2): threads take fixed segments of the rows for a pair of
+// columns each, every load of a chunk in flight, then the segments are added in order, so any
+// block computes the same totals.  res: ld entries; tmp: shared scratch of 2 * blockDim.x.
+__device__ __forceinline__ void colsum_rows(const float2* part, int G, int ld, float2* res,
+                                            float2* tmp) {
   const int bd = blockDim.x;
-  if (ld <= bd) {
-    const int nseg = bd / ld;
+  const int half = ld >> 1;  // column pairs: one float4 of two float-pairs per load
+  if (half <= bd) {
+    constexpr int CHUNK = 20;
+    const int nseg = bd / half;
     const int per = (G + nseg - 1) / nseg;
-    const int seg = threadIdx.x / ld, c = threadIdx.x % ld;
+    const int seg = threadIdx.x / half, cp = threadIdx.x % half;
     if (seg < nseg) {
       const int k0 = seg * per, k1 = min(G, k0 + per);
-      float2 acc = make_float2(0.f, 0.f);
-      for (int k = k0; k < k1; k += 8) {
-        float2 v[8];
+      float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
+      for (int k = k0; k < k1; k += CHUNK) {
+        float4 v[CHUNK];
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
-          v[j] = k + j < k1 ? __ldcg(cr.part1 + (size_t)(k + j) * ld + c) : make_float2(0.f, 0.f);
+        for (int j = 0; j < CHUNK; ++j)
+          v[j] = k + j < k1
+                     ? __ldcg(reinterpret_cast<const float4*>(part + (size_t)(k + j) * ld) + cp)
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc = df_add(acc, v[j]);
+        for (int j = 0; j < CHUNK; ++j) {
+          a0 = df_add(a0, make_float2(v[j].x, v[j].y));
+          a1 = df_add(a1, make_float2(v[j].z, v[j].w));
+        }
       }
-      tmp[seg * ld + c] = acc;
+      tmp[seg * ld + 2 * cp] = a0;
+      tmp[seg * ld + 2 * cp + 1] = a1;
     }
     __syncthreads();
-    if (threadIdx.x < ld) {
+    for (int c = threadIdx.x; c < ld; c += bd) {
       float2 acc = make_float2(0.f, 0.f);
-      for (int s = 0; s < nseg; ++s) acc = df_add(acc, tmp[s * ld + threadIdx.x]);
-      res[threadIdx.x] = acc;
+      for (int s = 0; s < nseg; ++s) acc = df_add(acc, tmp[s * ld + c]);
+      res[c] = acc;
     }
   } else {
     for (int c = threadIdx.x; c < ld; c += bd) {
@@ -229,16 +229,14 @@ __device__ __forceinline__ bool grid_colreduce_flat(const ColReduce& cr, const f
         float2 v[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j)
-          v[j] = k + j < G ? __ldcg(cr.part1 + (size_t)(k + j) * ld + c) : make_float2(0.f, 0.f);
+          v[j] = k + j < G ? __ldcg(part + (size_t)(k + j) * ld + c) : make_float2(0.f, 0.f);
 #pragma unroll
         for (int j = 0; j < 8; ++j) acc = df_add(acc, v[j]);
       }
       res[c] = acc;
     }
   }
-  if (threadIdx.x == 0) cr.cnt[0] = 0;
   __syncthreads();
-  return true;
 }
 
 // ------------------------------------------------------------------------------------------------

@@ -218,7 +218,8 @@ def erc_batched_cg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
 
 
 def erc_batched_cg_timed(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
-    """erc_batched_cg plus (solve microseconds, path): path 1 = resident single-launch solver."""
+    """erc_batched_cg plus (solve microseconds, path): 2 = cluster column-group solver, 1 = resident
+    cooperative solver, 0 = multi-kernel graph loop."""
     n, ld = Y.shape
     dev = Y.device
     X = torch.empty_like(Y) if X is None else X

@@ -45,11 +45,16 @@ def test_cg_matches_oracle_cg(kc):
     assert np.all(host(X)[:, kc:] == 0)
 
 
-@pytest.mark.parametrize("mode", ["graph", "auto"])
+PATHS = {"graph": 0, "resident": 1, "cluster": 2}
+
+
+@pytest.mark.parametrize("mode", list(PATHS))
 @pytest.mark.parametrize("kc,weighted,heavy", [(16, True, False), (128, False, False),
-                                               (64, True, True), (256, False, False)])
+                                               (64, True, True), (256, False, False),
+                                               (12, True, False)])
 def test_cg_paths_match_oracle(monkeypatch, mode, kc, weighted, heavy):
-    """The multi-kernel path and the resident single-launch path against the oracle."""
+    """Each solver path (multi-kernel graph, cooperative resident, cluster column groups)
+    against the oracle."""
     monkeypatch.setenv("ERC_CG_MODE", mode)
     n, src, dst, w = synth.random_connected(4000, 16000, seed=kc, weighted=weighted)
     if heavy:  # attach a hub to 3000 nodes so the block-split rows are exercised
@@ -60,8 +65,9 @@ def test_cg_paths_match_oracle(monkeypatch, mode, kc, weighted, heavy):
             w = np.concatenate([w, np.full(3000, 0.75, np.float32)])
     g, ref = build_both(n, src, dst, w)
     Y = erc.erc_jl_rhs(g, 9, 256, 0, kc)
-    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, kc, 1e-6)
+    X, iters, relres, st, _, path = erc.erc_batched_cg_timed(g, 1e-3, Y, kc, 1e-6)
     assert st == erc.ERC_OK
+    assert path == PATHS[mode]
     Xr, itr, _, _ = O.batched_cg(ref, 1e-3, O.jl_rhs(ref, 9, 256, 0, kc), 1e-6)
     Rg = torch.zeros(g.m, device=dev())
     erc.erc_edge_resistance(g, X, kc, Rg)
