@@ -625,7 +625,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   float2* part_rr = a.cr.part1 + (size_t)G * ld;       // [G][ld] block partials of r.r
   unsigned* arrivals = va.gen;
   // per-column CG state, the same in every block
-  __shared__ double s_rr[RMAXLD], s_yy[RMAXLD];
+  __shared__ float2 s_rr[RMAXLD], s_yy[RMAXLD];  // float pairs
   __shared__ __align__(16) float s_alpha[RMAXLD], s_beta[RMAXLD];
   __shared__ __align__(16) int s_active[RMAXLD];
   __shared__ int s_iters[RMAXLD], s_conv[RMAXLD];
@@ -637,8 +637,8 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   }
   int any = 0;
   for (int c = threadIdx.x; c < ld; c += PT) {
-    s_rr[c] = __ldcg(va.rr + c);
-    s_yy[c] = __ldcg(va.yy + c);
+    s_rr[c] = df_from_double(__ldcg(va.rr + c));
+    s_yy[c] = df_from_double(__ldcg(va.yy + c));
     s_alpha[c] = 0.f;
     s_beta[c] = 0.f;
     s_active[c] = __ldcg(va.active + c);
@@ -753,15 +753,15 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     res_wait(arrivals, ++nsync * G, va.flags);
     colsum_rows(part_pap, G, ld, sbuf, scratch);
     for (int c = threadIdx.x; c < ld; c += PT) {
-      const double v = df_value(sbuf[c]);
+      const float2 v = sbuf[c];
       float al = 0.f;
       if (s_active[c]) {
-        const double q = s_rr[c] / v;
-        if (!(v > 0.0) || !isfinite(q)) {
+        const float q = df_div(s_rr[c], v);
+        if (!(v.x > 0.f) || !isfinite(q)) {
           s_active[c] = 0;
           if (blockIdx.x == 0) atomicOr(&va.flags[1], 1);
         } else {
-          al = (float)q;
+          al = q;
         }
       }
       s_alpha[c] = al;
@@ -823,16 +823,16 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
       float be = 0.f;
       int act = s_active[c];
       if (act) {
-        const double rn = df_value(sbuf[c]);
+        const float2 rn = sbuf[c];
         const int it = s_iters[c] + 1;
         s_iters[c] = it;
-        if (!isfinite(rn)) {
+        if (!isfinite(rn.x)) {
           act = 0;
           if (blockIdx.x == 0) atomicOr(&va.flags[1], 1);
         } else {
-          be = (float)(rn / s_rr[c]);
+          be = df_div(rn, s_rr[c]);
           s_rr[c] = rn;
-          if (rn <= va.tol2 * s_yy[c]) {
+          if (df_value(rn) <= va.tol2 * df_value(s_yy[c])) {
             s_conv[c] = 1;
             act = 0;
           } else if (it >= va.max_iter) {
@@ -887,7 +887,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   // the per-column results, identical in every block
   if (blockIdx.x == 0)
     for (int c = threadIdx.x; c < ld; c += PT) {
-      va.rr[c] = s_rr[c];
+      va.rr[c] = df_value(s_rr[c]);
       va.iters[c] = s_iters[c];
       va.conv[c] = s_conv[c];
       va.active[c] = s_active[c];

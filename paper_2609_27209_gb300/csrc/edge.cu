@@ -16,14 +16,16 @@ __device__ __forceinline__ float4 ld_f4(const float* p) {
   return __ldg(reinterpret_cast<const float4*>(p));
 }
 
-// One group of LPR lanes walks a segment of consecutive canonical edges.  Edges are sorted by
-// their smaller endpoint, so X_u is reloaded only when u changes; the group owns each R_e it
-// touches, so the accumulation needs no atomics.
+// One group of LPR lanes walks a segment of consecutive canonical edges, EB edges at a time with
+// every row load of the batch issued before the first use.  Edges are sorted by their smaller
+// endpoint, so the X_u loads of a batch mostly hit L1.  The group owns each R_e it touches, so
+// the accumulation needs no atomics; per edge the column order and the lane tree are fixed.
 template <int LPR, int VPL>
 __global__ void __launch_bounds__(T)
     k_edge_resistance(const int32_t* __restrict__ eu, const int32_t* __restrict__ ev, int64_t m,
                       const float* __restrict__ X, int32_t ld, int32_t kc, float* __restrict__ R) {
   constexpr int SEG = 32;
+  constexpr int EB = VPL >= 4 ? 1 : 4 / VPL;
   const int gl = threadIdx.x & (LPR - 1);
   const int gpb = T / LPR;
   const int nvec = ld >> 2;
@@ -32,65 +34,82 @@ __global__ void __launch_bounds__(T)
   for (int64_t sg = (int64_t)blockIdx.x * gpb + threadIdx.x / LPR; sg < nseg;
        sg += (int64_t)gridDim.x * gpb) {
     const int64_t e0 = sg * SEG, e1 = min(m, e0 + SEG);
-    int32_t cu = -1;
-    float4 xu[VPL];
-    for (int64_t e = e0; e < e1; ++e) {
-      const int32_t u = __ldg(eu + e), v = __ldg(ev + e);
-      if (u != cu) {
+    for (int64_t eb = e0; eb < e1; eb += EB) {
+      float4 xu[EB][VPL], xv[EB][VPL];
+      float rold[EB];
 #pragma unroll
-        for (int k = 0; k < VPL; ++k) {
-          const int q = gl + LPR * k;
-          xu[k] = q < nvec ? ld_f4(X + (size_t)u * ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < EB; ++k) {
+        const bool ok = eb + k < e1;
+        const int32_t u = ok ? __ldg(eu + eb + k) : 0, v = ok ? __ldg(ev + eb + k) : 0;
+#pragma unroll
+        for (int t = 0; t < VPL; ++t) {
+          const int q = gl + LPR * t;
+          const bool on = ok && q < nvec;
+          xu[k][t] = on ? ld_f4(X + (size_t)u * ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
+          xv[k][t] = on ? ld_f4(X + (size_t)v * ld + 4 * q) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        cu = u;
+        rold[k] = ok && gl == 0 ? R[eb + k] : 0.f;
       }
-      float s = 0.f;
 #pragma unroll
-      for (int k = 0; k < VPL; ++k) {
-        const int q = gl + LPR * k;
-        if (q < nvec) {
-          const float4 xv = ld_f4(X + (size_t)v * ld + 4 * q);
-          const int cb = 4 * q;
-          const float dx = cb + 0 < kc ? xu[k].x - xv.x : 0.f;
-          const float dy = cb + 1 < kc ? xu[k].y - xv.y : 0.f;
-          const float dz = cb + 2 < kc ? xu[k].z - xv.z : 0.f;
-          const float dw = cb + 3 < kc ? xu[k].w - xv.w : 0.f;
+      for (int k = 0; k < EB; ++k) {
+        float s = 0.f;
+#pragma unroll
+        for (int t = 0; t < VPL; ++t) {
+          const int cb = 4 * (gl + LPR * t);
+          const float dx = cb + 0 < kc ? xu[k][t].x - xv[k][t].x : 0.f;
+          const float dy = cb + 1 < kc ? xu[k][t].y - xv[k][t].y : 0.f;
+          const float dz = cb + 2 < kc ? xu[k][t].z - xv[k][t].z : 0.f;
+          const float dw = cb + 3 < kc ? xu[k][t].w - xv[k][t].w : 0.f;
           s = fmaf(dx, dx, s);
           s = fmaf(dy, dy, s);
           s = fmaf(dz, dz, s);
           s = fmaf(dw, dw, s);
         }
-      }
 #pragma unroll
-      for (int off = LPR / 2; off > 0; off >>= 1) s += __shfl_xor_sync(gm, s, off, LPR);
-      if (gl == 0) R[e] += s;
+        for (int off = LPR / 2; off > 0; off >>= 1) s += __shfl_xor_sync(gm, s, off, LPR);
+        if (gl == 0 && eb + k < e1) R[eb + k] = rold[k] + s;
+      }
     }
   }
 }
 
-__device__ __forceinline__ double warp_sum(double v) {
+
+// Row sums of the node kernels: NL lanes per row, each adding its slots in a float pair, then a
+// fixed lane tree.  Float pairs keep about 44 bits without float64 arithmetic.
+constexpr int NL = 8;
+
+__device__ __forceinline__ float2 group_df_sum(float2 acc, unsigned gm) {
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-  return v;
+  for (int off = NL / 2; off > 0; off >>= 1) {
+    float2 o;
+    o.x = __shfl_xor_sync(gm, acc.x, off, NL);
+    o.y = __shfl_xor_sync(gm, acc.y, off, NL);
+    acc = df_add(acc, o);
+  }
+  return acc;
 }
 
-// p_u = 1 - 1/2 sum_{slots j of row u} w_j R[eid_j]; a warp per row, float64 sums
+// p_u = 1 - 1/2 sum_{slots j of row u} w_j R[eid_j] (Eq. 2), rounded once to float
+inline int node_grid(int32_t n) { return (int)(((int64_t)n + T / NL - 1) / (T / NL)); }
+
 template <bool WEIGHTED>
 __global__ void __launch_bounds__(T)
     k_node_curvature(const int64_t* __restrict__ row_ptr, const float* __restrict__ val,
                      const int32_t* __restrict__ eid, const float* __restrict__ R, int32_t n,
                      float* __restrict__ p) {
-  const int lane = threadIdx.x & 31;
-  const int64_t wpb = T / 32;
-  for (int64_t u = (int64_t)blockIdx.x * wpb + threadIdx.x / 32; u < n;
-       u += (int64_t)gridDim.x * wpb) {
-    double acc = 0.0;
-    for (int64_t j = row_ptr[u] + lane; j < row_ptr[u + 1]; j += 32) {
-      const double r = (double)__ldg(R + __ldg(eid + j));
-      acc += WEIGHTED ? (double)__ldg(val + j) * r : r;
-    }
-    acc = warp_sum(acc);
-    if (lane == 0) p[u] = (float)(1.0 - 0.5 * acc);
+  const int gl = threadIdx.x & (NL - 1);
+  const unsigned gm = group_mask<NL>();
+  const int64_t u = (int64_t)blockIdx.x * (T / NL) + threadIdx.x / NL;
+  if (u >= n) return;  // whole groups leave together: the grid covers every row once
+  float2 acc = make_float2(0.f, 0.f);
+  for (int64_t j = row_ptr[u] + gl; j < row_ptr[u + 1]; j += NL) {
+    const float r = __ldg(R + __ldg(eid + j));
+    acc = WEIGHTED ? df_fma(acc, __ldg(val + j), r) : df_add(acc, make_float2(r, 0.f));
+  }
+  acc = group_df_sum(acc, gm);
+  if (gl == 0) {  // 1 - acc / 2 as a pair, then rounded
+    const float2 s = df_two_sum(1.f, -0.5f * acc.x);
+    p[u] = __fadd_rn(s.x, __fsub_rn(s.y, 0.5f * acc.y));
   }
 }
 
@@ -181,27 +200,31 @@ __global__ void __launch_bounds__(T) k_minmax_final(const float* part_min, const
   }
 }
 
-// Eq. 7 row sums: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta)
+// Eq. 7 row sums: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta).
+// Each difference kappa - kappa_min is exact as a float pair; the row's pair sum is scaled once
+// in float64.  Per block: the sum of q_u and the number of non-isolated nodes.
 __global__ void __launch_bounds__(T)
     k_qnode(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ eid,
             const float* __restrict__ kappa, int32_t n, double eta, const double* scal,
             double* __restrict__ qnode, double* part_qn, double* part_cnt) {
   __shared__ double sh[T];
-  const int lane = threadIdx.x & 31;
-  const int64_t wpb = T / 32;
-  const double kmin = scal[0];
+  const int gl = threadIdx.x & (NL - 1);
+  const unsigned gm = group_mask<NL>();
+  const float kmin = (float)scal[0];  // the minimum of float kappa: exact
   const double inv = 1.0 / (scal[1] - scal[0] + eta);
   double tq = 0.0, tc = 0.0;
-  for (int64_t u = (int64_t)blockIdx.x * wpb + threadIdx.x / 32; u < n;
-       u += (int64_t)gridDim.x * wpb) {
+  for (int64_t u = (int64_t)blockIdx.x * (T / NL) + threadIdx.x / NL; u < n;
+       u += (int64_t)gridDim.x * (T / NL)) {  // the same trip count for a group's lanes
     const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
-    double acc = 0.0;
-    for (int64_t j = j0 + lane; j < j1; j += 32) acc += ((double)__ldg(kappa + __ldg(eid + j)) - kmin) * inv;
-    acc = warp_sum(acc);
-    if (lane == 0) {
-      qnode[u] = acc;
-      tq += acc;
-      tc += (j1 > j0) ? 1.0 : 0.0;
+    float2 acc = make_float2(0.f, 0.f);
+    for (int64_t j = j0 + gl; j < j1; j += NL)
+      acc = df_add(acc, df_two_sum(__ldg(kappa + __ldg(eid + j)), -kmin));
+    acc = group_df_sum(acc, gm);
+    if (gl == 0) {
+      const double q = df_value(acc) * inv;
+      qnode[u] = q;
+      tq += q;
+      tc += j1 > j0 ? 1.0 : 0.0;
     }
   }
   tq = block_reduce(tq, AddD{}, sh);
@@ -302,10 +325,10 @@ extern "C" erc_status erc_curvature(const erc_graph* g, const float* R, float* p
   ERC_REQUIRE(p_node && (kappa || g->m == 0) && (R || g->m == 0), "R, p_node, kappa required");
   cudaStream_t s = as_stream(stream);
   if (g->val)
-    k_node_curvature<true><<<grid_for(g->n, T / 32), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
+    k_node_curvature<true><<<node_grid(g->n), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
                                                                 R, g->n, p_node);
   else
-    k_node_curvature<false><<<grid_for(g->n, T / 32), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
+    k_node_curvature<false><<<node_grid(g->n), T, 0, s>>>(g->row_ptr, g->val, g->csr_eid,
                                                                  R, g->n, p_node);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
@@ -350,7 +373,7 @@ extern "C" erc_status erc_sampling_probs(const erc_graph* g, const float* kappa,
   k_minmax_final<<<1, T, 0, s>>>(w.part_min, w.part_max, ge, w.scal);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
-  const int gn = grid_for(g->n, T / 32);
+  const int gn = grid_for(g->n, T / NL);
   k_qnode<<<gn, T, 0, s>>>(g->row_ptr, g->csr_eid, kappa, g->n, (double)eta, w.scal, w.qnode,
                            w.part_qn, w.part_cnt);
   count_launches(1);

@@ -90,6 +90,18 @@ __device__ __forceinline__ float2 df_fma(float2 acc, float a, float b) {
   return df_norm(s.x, __fadd_rn(s.y, __fadd_rn(acc.y, pe)));
 }
 __device__ __forceinline__ double df_value(float2 a) { return (double)a.x + (double)a.y; }
+__device__ __forceinline__ float2 df_from_double(double v) {
+  const float hi = (float)v;
+  return make_float2(hi, (float)(v - (double)hi));
+}
+// (a.x + a.y) / (b.x + b.y) rounded to float, without float64 arithmetic: Dekker's pair division
+// (T. J. Dekker, "A floating-point technique for extending the available precision", 1971) with
+// one correction step.  q0 b.x is subtracted exactly by the fused multiply-add.
+__device__ __forceinline__ float df_div(float2 a, float2 b) {
+  const float q0 = __fdiv_rn(a.x, b.x);
+  const float r = __fadd_rn(__fmaf_rn(-q0, b.x, a.x), a.y);
+  return __fadd_rn(q0, __fdiv_rn(__fmaf_rn(-q0, b.y, r), b.x));
+}
 
 // ------------------------------------------------------------------------------------------------
 // deterministic grid-wide per-column reduction of float2 partials.

@@ -23,50 +23,77 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   return c;
 }
 
-// the 32-bit Philox word holding the sign bits of columns 32*(c/32) .. +31 of edge e
-__device__ __forceinline__ uint32_t sign_word(uint2 key, uint32_t e, int c, int& cached_g,
-                                              uint4& cached) {
-  const int g = c >> 7;
-  if (g != cached_g) {
-    cached = philox4x32_10(make_uint4((uint32_t)g, 0u, e, 0u), key);
-    cached_g = g;
-  }
-  const int wi = (c >> 5) & 3;
-  return wi == 0 ? cached.x : wi == 1 ? cached.y : wi == 2 ? cached.z : cached.w;
-}
-
+// Row u of Y: the LPR lanes of a group walk u's CSR slots LPR at a time.  Lane l generates the
+// Philox blocks of slot jb + l (one per 128-column block its group covers) and the slot's signed
+// coefficient; the slots are then applied in CSR order, each lane taking from the generating
+// lane, by shuffles, the word that holds its four columns' sign bits.
 template <int LPR, int VPL, bool WEIGHTED>
 __global__ void __launch_bounds__(256)
     k_jl_rhs(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ col,
              const float* __restrict__ val, const int32_t* __restrict__ csr_eid, int32_t n,
              uint2 key, float inv_sqrt_k, int32_t c0, int32_t kc, int32_t ld, float* __restrict__ Y) {
+  constexpr int NBM = VPL + 1;  // 128-column Philox blocks a group's columns can span
   const int gl = threadIdx.x & (LPR - 1);
+  const unsigned gm = group_mask<LPR>();
   const int groups_per_block = blockDim.x / LPR;
   const int64_t ngroups = (int64_t)gridDim.x * groups_per_block;
   const int nvec = ld >> 2;
+  const int g0 = c0 >> 7;
+  const int nb = ((c0 + 4 * (nvec - 1)) >> 7) - g0 + 1;
+  int blk[VPL], wsel[VPL], sh[VPL];
+  bool on[VPL];
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int q = gl + LPR * v;
+    const int c = c0 + 4 * q;  // c0 % 4 == 0: the four columns share one word
+    on[v] = q < nvec && 4 * q < kc;
+    blk[v] = (c >> 7) - g0;
+    wsel[v] = (c >> 5) & 3;
+    sh[v] = c & 31;
+  }
   for (int64_t u = (int64_t)blockIdx.x * groups_per_block + threadIdx.x / LPR; u < n;
        u += ngroups) {
     float4 acc[VPL];
 #pragma unroll
     for (int v = 0; v < VPL; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
     const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
-    for (int64_t j = j0; j < j1; ++j) {
-      const int32_t nb = col[j];
-      const uint32_t e = (uint32_t)csr_eid[j];
-      float coef = WEIGHTED ? sqrtf(val[j]) * inv_sqrt_k : inv_sqrt_k;
-      if (nb < u) coef = -coef;  // u is the larger endpoint: row e of B is e_nb - e_u
-      int cg = -1;
-      uint4 cw;
+    for (int64_t jb = j0; jb < j1; jb += LPR) {
+      const int64_t j = jb + gl;
+      float coef = 0.f;
+      uint4 w[NBM];
 #pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        if (q < nvec && 4 * q < kc) {
-          const int c = c0 + 4 * q;  // c0 % 4 == 0: the four columns share one word
-          const uint32_t bits = sign_word(key, e, c, cg, cw) >> (c & 31);
-          acc[v].x += (bits & 1u) ? -coef : coef;
-          acc[v].y += (bits & 2u) ? -coef : coef;
-          acc[v].z += (bits & 4u) ? -coef : coef;
-          acc[v].w += (bits & 8u) ? -coef : coef;
+      for (int b = 0; b < NBM; ++b) w[b] = make_uint4(0u, 0u, 0u, 0u);
+      if (j < j1) {
+        const uint32_t e = (uint32_t)csr_eid[j];
+        coef = WEIGHTED ? sqrtf(val[j]) * inv_sqrt_k : inv_sqrt_k;
+        if (col[j] < u) coef = -coef;  // u is the larger endpoint: row e of B is e_nb - e_u
+#pragma unroll
+        for (int b = 0; b < NBM; ++b)
+          if (b < nb) w[b] = philox4x32_10(make_uint4((uint32_t)(g0 + b), 0u, e, 0u), key);
+      }
+      const int cnt = (int)min((int64_t)LPR, j1 - jb);
+      for (int k = 0; k < cnt; ++k) {
+        const float cf = __shfl_sync(gm, coef, k, LPR);
+        uint32_t word[VPL];
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) word[v] = 0u;
+#pragma unroll
+        for (int b = 0; b < NBM; ++b) {
+          if (b >= nb) break;
+          const uint32_t x = __shfl_sync(gm, w[b].x, k, LPR), y = __shfl_sync(gm, w[b].y, k, LPR);
+          const uint32_t z = __shfl_sync(gm, w[b].z, k, LPR), t = __shfl_sync(gm, w[b].w, k, LPR);
+#pragma unroll
+          for (int v = 0; v < VPL; ++v)
+            if (blk[v] == b) word[v] = wsel[v] == 0 ? x : wsel[v] == 1 ? y : wsel[v] == 2 ? z : t;
+        }
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) {
+          if (!on[v]) continue;
+          const uint32_t bits = word[v] >> sh[v];
+          acc[v].x += (bits & 1u) ? -cf : cf;
+          acc[v].y += (bits & 2u) ? -cf : cf;
+          acc[v].z += (bits & 4u) ? -cf : cf;
+          acc[v].w += (bits & 8u) ? -cf : cf;
         }
       }
     }
