@@ -14,13 +14,97 @@ namespace erc {
 namespace {
 thread_local char g_err[512] = "";
 thread_local bool g_capturing = false;
+thread_local long long g_captured = 0;  // kernels recorded into the graph being captured
 std::atomic<unsigned long long> g_launches{0};
 }
 
 void count_launches(long long k) {
-  if (!g_capturing) g_launches.fetch_add((unsigned long long)k, std::memory_order_relaxed);
+  if (g_capturing)
+    g_captured += k;
+  else
+    g_launches.fetch_add((unsigned long long)k, std::memory_order_relaxed);
 }
-void set_capturing(bool on) { g_capturing = on; }
+void set_capturing(bool on) {
+  g_capturing = on;
+  if (on) g_captured = 0;
+}
+
+// ---- cached launch sequences (see GraphKey)
+namespace {
+struct CachedGraph {
+  GraphKey key;
+  cudaGraphExec_t exec = nullptr;
+  long long kernels = 0;
+  unsigned long long stamp = 0;
+};
+constexpr int GRAPHS = 32;
+std::mutex g_graph_mu;
+CachedGraph g_graphs[GRAPHS];
+unsigned long long g_graph_clock = 0;
+
+bool same_key(const GraphKey& a, const GraphKey& b) {
+  if (a.n != b.n) return false;
+  for (int i = 0; i < a.n; ++i)
+    if (a.w[i] != b.w[i]) return false;
+  return true;
+}
+
+cudaStream_t private_stream() {
+  static thread_local cudaStream_t cs[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!cs[dev] && cudaStreamCreateWithFlags(&cs[dev], cudaStreamNonBlocking) != cudaSuccess)
+    return nullptr;
+  return cs[dev];
+}
+}  // namespace
+
+erc_status graph_launch_impl(const GraphKey& key_in, erc_status (*enqueue)(void*, cudaStream_t),
+                             void* ctx, cudaStream_t s) {
+  GraphKey key = key_in;
+  int dev = 0;
+  ERC_CUDA(cudaGetDevice(&dev));
+  key.add((uint64_t)dev);
+  std::lock_guard<std::mutex> lock(g_graph_mu);
+  ++g_graph_clock;
+  int victim = 0;
+  for (int i = 0; i < GRAPHS; ++i) {
+    if (g_graphs[i].exec && same_key(g_graphs[i].key, key)) {
+      g_graphs[i].stamp = g_graph_clock;
+      ERC_CUDA(cudaGraphLaunch(g_graphs[i].exec, s));
+      count_launches(g_graphs[i].kernels);
+      return ERC_OK;
+    }
+    if (g_graphs[i].stamp < g_graphs[victim].stamp) victim = i;
+  }
+  cudaStream_t cs = private_stream();
+  if (!cs) return set_error(ERC_ERR_CUDA, "no capture stream");
+  ERC_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  set_capturing(true);
+  const erc_status st = enqueue(ctx, cs);
+  const long long kernels = g_captured;
+  set_capturing(false);
+  cudaGraph_t graph = nullptr;
+  const cudaError_t ce = cudaStreamEndCapture(cs, &graph);
+  if (st != ERC_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return st;
+  }
+  if (ce != cudaSuccess) return set_error(ERC_ERR_CUDA, "graph capture: %s", cudaGetErrorString(ce));
+  cudaGraphExec_t exec = nullptr;
+  const cudaError_t ie = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (ie != cudaSuccess)
+    return set_error(ERC_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(ie));
+  if (g_graphs[victim].exec) cudaGraphExecDestroy(g_graphs[victim].exec);
+  g_graphs[victim].key = key;
+  g_graphs[victim].exec = exec;
+  g_graphs[victim].kernels = kernels;
+  g_graphs[victim].stamp = g_graph_clock;
+  ERC_CUDA(cudaGraphLaunch(exec, s));
+  count_launches(kernels);
+  return ERC_OK;
+}
 
 erc_status set_error(erc_status code, const char* fmt, ...) {
   va_list ap;

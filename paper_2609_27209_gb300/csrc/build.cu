@@ -206,45 +206,55 @@ extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const i
   BuildPlan p;
   plan_build(a, p, m_in);
 
-  ERC_CUDA(cudaMemsetAsync(p.counters, 0, 4 * sizeof(int64_t), s));
-  ERC_CUDA(cudaMemsetAsync(p.err, 0, 4 * sizeof(unsigned), s));
-  ERC_CUDA(cudaMemsetAsync(row_ptr, 0, (size_t)(n + 1) * sizeof(int64_t), s));
+  // the launch sequence is replayed from a cached CUDA graph: some twenty small kernels whose
+  // launch overhead would otherwise exceed their run time
   const int64_t E = 2 * m_in;
   const int B = bit_length((uint32_t)n);  // 2^B > n - 1: every id fits, and the sentinel sorts last
   const uint64_t sent = (2 * B >= 64) ? ~0ull : ((1ull << (2 * B)) - 1ull);
-  if (m_in > 0) {
-    k_emit<<<grid_for(m_in, BT), BT, 0, s>>>(src, dst, w, m_in, n, B, sent, p.keys, p.vals, p.err);
+  auto enqueue = [&](cudaStream_t cs) -> erc_status {
+    ERC_CUDA(cudaMemsetAsync(p.counters, 0, 4 * sizeof(int64_t), cs));
+    ERC_CUDA(cudaMemsetAsync(p.err, 0, 4 * sizeof(unsigned), cs));
+    ERC_CUDA(cudaMemsetAsync(row_ptr, 0, (size_t)(n + 1) * sizeof(int64_t), cs));
+    if (m_in > 0) {
+      k_emit<<<grid_for(m_in, BT), BT, 0, cs>>>(src, dst, w, m_in, n, B, sent, p.keys, p.vals,
+                                                p.err);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+      ERC_TRY(radix_sort_pairs(p.keys, p.vals, p.keys_alt, p.vals_alt, E, 2 * B, p.sort_tmp, cs));
+      k_heads<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, E, sent, p.head);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+      ERC_TRY(exclusive_scan_i64(nullptr, p.head, p.slot, E, &p.counters[0], p.scan_tmp, cs));
+      ERC_CUDA(cudaMemsetAsync(p.upper, 0, (size_t)E, cs));  // slots past nnz must not count
+      k_emit_csr<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, p.vals, p.head, p.slot, w, E, B,
+                                                dup_policy == ERC_DUP_FIRST, col, p.wmerged,
+                                                p.row_of, p.upper);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+      k_row_ptr<<<grid_for(E, BT), BT, 0, cs>>>(p.row_of, p.counters, n, row_ptr);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+    }
+    k_degree<<<grid_for(n, BT), BT, 0, cs>>>(row_ptr, p.wmerged, n, deg, val, p.counters);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
-    ERC_TRY(radix_sort_pairs(p.keys, p.vals, p.keys_alt, p.vals_alt, E, 2 * B, p.sort_tmp, s));
-    k_heads<<<grid_for(E, BT), BT, 0, s>>>(p.keys, E, sent, p.head);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    ERC_TRY(exclusive_scan_i64(nullptr, p.head, p.slot, E, &p.counters[0], p.scan_tmp, s));
-    ERC_CUDA(cudaMemsetAsync(p.upper, 0, (size_t)E, s));  // slots past nnz must not count
-    k_emit_csr<<<grid_for(E, BT), BT, 0, s>>>(p.keys, p.vals, p.head, p.slot, w, E, B,
-                                              dup_policy == ERC_DUP_FIRST, col, p.wmerged,
-                                              p.row_of, p.upper);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    k_row_ptr<<<grid_for(E, BT), BT, 0, s>>>(p.row_of, p.counters, n, row_ptr);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-  }
-  k_degree<<<grid_for(n, BT), BT, 0, s>>>(row_ptr, p.wmerged, n, deg, val, p.counters);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-  if (m_in > 0) {
-    ERC_TRY(exclusive_scan_i64(nullptr, p.upper, p.eidx, E, &p.counters[1], p.scan_tmp, s));
-    k_emit_edges<<<grid_for(E, BT), BT, 0, s>>>(p.upper, p.eidx, p.row_of, col, p.wmerged,
-                                                p.counters, eu, ev, ew, csr_eid);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    k_lower_eid<<<grid_for(E, BT), BT, 0, s>>>(p.upper, p.row_of, col, row_ptr, p.counters,
-                                               csr_eid);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-  }
+    if (m_in > 0) {
+      ERC_TRY(exclusive_scan_i64(nullptr, p.upper, p.eidx, E, &p.counters[1], p.scan_tmp, cs));
+      k_emit_edges<<<grid_for(E, BT), BT, 0, cs>>>(p.upper, p.eidx, p.row_of, col, p.wmerged,
+                                                  p.counters, eu, ev, ew, csr_eid);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+      k_lower_eid<<<grid_for(E, BT), BT, 0, cs>>>(p.upper, p.row_of, col, row_ptr, p.counters,
+                                                 csr_eid);
+      count_launches(1);
+      ERC_CUDA(cudaGetLastError());
+    }
+    return ERC_OK;
+  };
+  GraphKey key;
+  key.add((uint64_t)n).add((uint64_t)m_in).add((uint64_t)dup_policy).add(src).add(dst).add(w);
+  key.add(row_ptr).add(col).add(val).add(deg).add(csr_eid).add(eu).add(ev).add(ew).add(a.base);
+  ERC_TRY(graph_launch(key, enqueue, s));
   int64_t h_counters[2] = {0, 0};
   unsigned h_err = 0;
   ERC_CUDA(cudaMemcpyAsync(h_counters, p.counters, 2 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));

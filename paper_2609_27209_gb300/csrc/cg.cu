@@ -1528,6 +1528,38 @@ const void* resident_kernel(int nvec, bool weighted) {
   return k;  // wider rows use the multi-kernel path
 }
 
+// Raise a kernel's dynamic shared-memory limit to everything the block may use, once per device
+// and kernel; each launch then asks for what its plan needs.  Returns the limit (0 on failure).
+size_t open_smem(const void* k) {
+  static std::mutex mu;
+  static const void* done_k[64][32] = {};
+  static size_t done_v[64][32] = {};
+  int dev = 0, optin = 0;
+  cudaFuncAttributes fa;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < 32; ++i)
+    if (done_k[dev][i] == k) return done_v[dev][i];
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+      cudaFuncGetAttributes(&fa, k) != cudaSuccess || (size_t)optin <= fa.sharedSizeBytes) {
+    cudaGetLastError();
+    return 0;
+  }
+  const size_t lim = (size_t)optin - fa.sharedSizeBytes;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lim) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  for (int i = 0; i < 32; ++i)
+    if (!done_k[dev][i]) {
+      done_k[dev][i] = k;
+      done_v[dev][i] = lim;
+      break;
+    }
+  return lim;
+}
+
 bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const void** kern) {
   const int nvec = ld / 4;
   const void* k = resident_kernel(nvec, g->val != nullptr);
@@ -1537,20 +1569,7 @@ bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const 
   const int64_t rows = ((int64_t)g->n + grid - 1) / grid;
   const size_t bytes = 4 * (2 * (size_t)rows * ld + (size_t)(PT / lpr) * ld + 2 * (size_t)ld +
                             2 * (size_t)PWARPS * PCH);
-  int dev = 0, optin = 0;
-  cudaFuncAttributes fa;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
-      cudaFuncGetAttributes(&fa, k) != cudaSuccess) {
-    cudaGetLastError();
-    return false;
-  }
-  if (bytes + fa.sharedSizeBytes > (size_t)optin) return false;
-  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) !=
-      cudaSuccess) {
-    cudaGetLastError();
-    return false;
-  }
+  if (bytes > open_smem(k)) return false;
   int nb = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, PT, bytes) != cudaSuccess || nb < 1) {
     cudaGetLastError();
@@ -1605,17 +1624,14 @@ void cluster_config(const ClusterPlan& pl, cudaStream_t s, cudaLaunchConfig_t* c
 
 bool cluster_plan(const erc_graph* g, int ld, ClusterPlan* pl) {
   const void* k = g->val ? (const void*)k_cg_cluster<true> : (const void*)k_cg_cluster<false>;
-  int dev = 0, optin = 0;
-  cudaFuncAttributes fa;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
-      cudaFuncGetAttributes(&fa, k) != cudaSuccess ||
-      cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+  const size_t lim = open_smem(k);
+  if (!lim || cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                  cudaSuccess) {
     cudaGetLastError();
     return false;
   }
   const int64_t row_bytes = 2 * CL * sizeof(float4);  // r and Ap of the group's columns
-  const int64_t cap = ((int64_t)optin - (int64_t)fa.sharedSizeBytes - 1024) / row_bytes;
+  const int64_t cap = ((int64_t)lim - 1024) / row_bytes;
   const int groups = (ld / 4 + CL - 1) / CL;
   for (int S = CMAXS; S >= 1; --S) {
     const int64_t even = ((int64_t)g->n + S - 1) / S;
@@ -1626,11 +1642,6 @@ bool cluster_plan(const erc_graph* g, int ld, ClusterPlan* pl) {
     p.groups = groups;
     p.rbmax = (int32_t)std::min(cap, even + even / 8 + 32);  // room to balance neighbour lists
     p.smem = (size_t)p.rbmax * row_bytes;
-    if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem) !=
-        cudaSuccess) {
-      cudaGetLastError();
-      continue;
-    }
     cudaLaunchConfig_t cfg;
     cudaLaunchAttribute attr[1];
     cluster_config(p, nullptr, &cfg, attr);
@@ -1644,6 +1655,48 @@ bool cluster_plan(const erc_graph* g, int ld, ClusterPlan* pl) {
     return true;
   }
   return false;
+}
+
+// Both single-launch plans for a graph shape, computed once per (device, n, ld, weighted): the
+// occupancy queries behind them cost more host time than a small solve.
+struct SolverPlans {
+  bool cluster = false, resident = false;
+  ClusterPlan cp;
+  int32_t rb = 0;
+  size_t smem = 0;
+  const void* kres = nullptr;
+};
+
+SolverPlans solver_plans(const erc_graph* g, int ld) {
+  struct Entry {
+    int dev = -1;
+    int32_t n = 0, ld = 0;
+    bool weighted = false;
+    SolverPlans p;
+  };
+  static std::mutex mu;
+  static Entry cache[16];
+  static int next = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const bool weighted = g->val != nullptr;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (const Entry& e : cache)
+      if (e.dev == dev && e.n == g->n && e.ld == ld && e.weighted == weighted) return e.p;
+  }
+  SolverPlans p;
+  p.cluster = cluster_plan(g, ld, &p.cp);
+  p.resident = resident_plan(g, ld, &p.rb, &p.smem, &p.kres);
+  std::lock_guard<std::mutex> lock(mu);
+  Entry& e = cache[next];
+  next = (next + 1) % 16;
+  e.dev = dev;
+  e.n = g->n;
+  e.ld = ld;
+  e.weighted = weighted;
+  e.p = p;
+  return p;
 }
 
 // Where both single-launch solvers fit, the cheaper per iteration by a model fitted to GB300
@@ -1862,12 +1915,13 @@ static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y,
   // path: 2 cluster (column groups), 1 resident (one cooperative launch), 0 multi-kernel graph.
   // ERC_CG_MODE=graph|resident|cluster restricts the choice (testing of every path).
   const char* mode = getenv("ERC_CG_MODE");
-  ClusterPlan cp;
-  bool cluster = (!mode || strcmp(mode, "cluster") == 0) && cluster_plan(g, ld, &cp);
-  int32_t rb = 0;
-  size_t smem = 0;
-  const void* kres = nullptr;
-  bool resident = (!mode || strcmp(mode, "resident") == 0) && resident_plan(g, ld, &rb, &smem, &kres);
+  const SolverPlans plans = solver_plans(g, ld);
+  const ClusterPlan& cp = plans.cp;
+  const int32_t rb = plans.rb;
+  const size_t smem = plans.smem;
+  const void* kres = plans.kres;
+  bool cluster = (!mode || strcmp(mode, "cluster") == 0) && plans.cluster;
+  bool resident = (!mode || strcmp(mode, "resident") == 0) && plans.resident;
   if (cluster && resident) {
     if (prefer_cluster(g, ld, cp))
       resident = false;

@@ -47,6 +47,31 @@ int sm_count();
 void count_launches(long long k);
 void set_capturing(bool on);
 
+// A launch sequence replayed as a CUDA graph: `enqueue` is captured once per key (on a private
+// stream of the current device) into an executable graph, kept in a small least-recently-used
+// cache, and launched on `s`.  The key must hold everything the sequence depends on: pointers,
+// sizes, scalars and the device.  Host reads of device results stay outside the sequence.
+struct GraphKey {
+  static constexpr int WORDS = 32;
+  uint64_t w[WORDS] = {};
+  int n = 0;
+  GraphKey& add(uint64_t v) {
+    if (n < WORDS) w[n++] = v;
+    return *this;
+  }
+  GraphKey& add(const void* p) { return add((uint64_t)(uintptr_t)p); }
+};
+template <class F>
+erc_status graph_launch(GraphKey key, F&& enqueue, cudaStream_t s);
+erc_status graph_launch_impl(const GraphKey& key, erc_status (*enqueue)(void*, cudaStream_t),
+                             void* ctx, cudaStream_t s);
+template <class F>
+erc_status graph_launch(GraphKey key, F&& enqueue, cudaStream_t s) {
+  using Fn = std::remove_reference_t<F>;
+  auto thunk = [](void* c, cudaStream_t cs) -> erc_status { return (*static_cast<Fn*>(c))(cs); };
+  return graph_launch_impl(key, thunk, const_cast<void*>(static_cast<const void*>(&enqueue)), s);
+}
+
 // ------------------------------------------------------------------------------------------------
 // workspace carving: the same plan runs once to size (base == nullptr) and once to carve
 // ------------------------------------------------------------------------------------------------
