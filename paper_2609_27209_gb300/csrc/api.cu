@@ -164,20 +164,11 @@ erc_status check_graph(const erc_graph* g) {
 
 namespace {
 
-__global__ void k_all_unit(const float* __restrict__ w, int64_t m, int* __restrict__ nonunit) {
-  int bad = 0;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < m;
-       e += (int64_t)gridDim.x * blockDim.x)
-    bad |= (w[e] != 1.f);
-  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(nonunit, 1);
-}
-
 struct RunPlan {
   int64_t* row_ptr;
   int32_t *col, *csr_eid;
   float *val, *deg, *ew;
   float *Y, *X;
-  int* flag;
   void* cg_ws;
   size_t cg_bytes;
   void* aux_ws;  // build workspace, later the sampling workspace
@@ -196,7 +187,6 @@ void plan_run(Arena& a, RunPlan& p, int32_t n, int64_t m_in, int32_t kc) {
   p.ew = a.take<float>(m_in);
   p.Y = a.take<float>((size_t)n * ld);
   p.X = a.take<float>((size_t)n * ld);
-  p.flag = a.take<int>(4);
   p.cg_bytes = erc_batched_cg_workspace_size(n, ld);
   p.cg_ws = a.take<char>(p.cg_bytes);
   const size_t b1 = erc_build_laplacian_workspace_size(n, m_in);
@@ -211,43 +201,29 @@ erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, cons
                       int32_t* iters, float* relres, const RunPlan& p, cudaStream_t s) {
   const int32_t ld = ld_for(prm->kc);
   int64_t m = 0;
-  ERC_TRY(erc_build_laplacian(n, src, dst, w, m_in, prm->dup_policy, p.row_ptr, p.col, p.val,
-                              p.deg, p.csr_eid, eu, ev, p.ew, &m, p.aux_ws, p.aux_bytes,
-                              reinterpret_cast<erc_stream>(s)));
-  *m_out = m;
-  // an unweighted input whose duplicates did not merge keeps unit weights: drop the weight
-  // arrays so the gathers read indices only
+  // the build also reports whether an unweighted input kept unit weights (no merged duplicates):
+  // then the weight arrays are dropped and the gathers read indices only
   int nonunit = 1;
-  if (!w && m > 0) {
-    ERC_CUDA(cudaMemsetAsync(p.flag, 0, sizeof(int), s));
-    k_all_unit<<<grid_for(m, 256), 256, 0, s>>>(p.ew, m, p.flag);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    ERC_CUDA(cudaMemcpyAsync(&nonunit, p.flag, sizeof(int), cudaMemcpyDeviceToHost, s));
-    ERC_CUDA(cudaStreamSynchronize(s));
-  }
+  ERC_TRY(build_laplacian_impl(n, src, dst, w, m_in, prm->dup_policy, p.row_ptr, p.col, p.val,
+                               p.deg, p.csr_eid, eu, ev, p.ew, &m, p.aux_ws, p.aux_bytes, s,
+                               &nonunit));
+  *m_out = m;
   erc_graph g{n, m, p.row_ptr, p.col, nonunit ? p.val : nullptr, p.deg, p.csr_eid,
               eu, ev, nonunit ? p.ew : nullptr};
   if (m > 0) ERC_CUDA(cudaMemsetAsync(R, 0, (size_t)m * sizeof(float), s));
-  erc_status worst = ERC_OK;
+  // every batch is enqueued without a host round trip (the single-launch solvers need none); the
+  // CG status of all batches is read once at the end
   for (int32_t c0 = 0; c0 < prm->K; c0 += prm->kc) {
     const int32_t k = prm->kc < prm->K - c0 ? prm->kc : prm->K - c0;
     ERC_TRY(erc_jl_rhs(&g, prm->seed, prm->K, c0, k, p.Y, ld, reinterpret_cast<erc_stream>(s)));
-    erc_status st = erc_batched_cg(&g, prm->eps, p.Y, p.X, ld, k, prm->tol, prm->max_iter,
-                                   iters + c0, relres + c0, p.cg_ws, p.cg_bytes,
-                                   reinterpret_cast<erc_stream>(s));
-    if (st == ERC_ERR_NOT_CONVERGED) {
-      worst = st;
-    } else if (st != ERC_OK) {
-      return st;
-    }
+    ERC_TRY(cg_enqueue(&g, prm->eps, p.Y, p.X, ld, k, prm->tol, prm->max_iter, iters + c0,
+                       relres + c0, p.cg_ws, p.cg_bytes, s, c0 == 0, nullptr, nullptr, nullptr));
     ERC_TRY(erc_edge_resistance(&g, p.X, ld, k, R, reinterpret_cast<erc_stream>(s)));
   }
   ERC_TRY(erc_curvature(&g, R, p_node, kappa, reinterpret_cast<erc_stream>(s)));
   ERC_TRY(erc_sampling_probs(&g, kappa, prm->eta, prob_node, prob_edge, p.aux_ws, p.aux_bytes,
                              reinterpret_cast<erc_stream>(s)));
-  if (worst != ERC_OK) return set_error(worst, "some CG columns reached max_iter");
-  return ERC_OK;
+  return cg_status(n, ld, prm->K, prm->max_iter, p.cg_ws, s);
 }
 
 erc_status check_params(const erc_params* prm, int32_t n, int64_t m_in) {

@@ -79,12 +79,16 @@ __global__ void k_heads(const uint64_t* __restrict__ keys, int64_t E, uint64_t s
   }
 }
 
+// nonunit (may be null): set to 1 when some merged weight differs from 1 (unweighted inputs with
+// merged duplicates)
 __global__ void k_emit_csr(const uint64_t* __restrict__ keys, const uint32_t* __restrict__ vals,
                            const uint8_t* __restrict__ head, const int64_t* __restrict__ slot,
                            const float* __restrict__ w, int64_t E, int B, int dup_first,
                            int32_t* __restrict__ col, float* __restrict__ wmerged,
-                           int32_t* __restrict__ row_of, uint8_t* __restrict__ upper) {
+                           int32_t* __restrict__ row_of, uint8_t* __restrict__ upper,
+                           unsigned* __restrict__ nonunit) {
   const uint64_t mask = (1ull << B) - 1ull;
+  bool other = false;
   for (int64_t i = gtid(); i < E; i += gstride()) {
     if (!head[i]) continue;
     const uint64_t k = keys[i];
@@ -101,7 +105,9 @@ __global__ void k_emit_csr(const uint64_t* __restrict__ keys, const uint32_t* __
     row_of[s] = r;
     wmerged[s] = (float)acc;
     upper[s] = c > r;
+    other |= (float)acc != 1.f;
   }
+  if (nonunit && __any_sync(0xffffffffu, other) && (threadIdx.x & 31) == 0) atomicOr(nonunit, 1u);
 }
 
 __global__ void k_row_ptr(const int32_t* __restrict__ row_of, const int64_t* __restrict__ counters,
@@ -182,14 +188,12 @@ extern "C" size_t erc_build_laplacian_workspace_size(int32_t n, int64_t m_in) {
   return a.used + 256;
 }
 
-extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const int32_t* dst,
-                                          const float* w, int64_t m_in, int32_t dup_policy,
-                                          int64_t* row_ptr, int32_t* col, float* val, float* deg,
-                                          int32_t* csr_eid, int32_t* eu, int32_t* ev, float* ew,
-                                          int64_t* m_out, void* ws, size_t ws_bytes,
-                                          erc_stream stream) {
-  clear_error();
-  cudaStream_t s = as_stream(stream);
+erc_status erc::build_laplacian_impl(int32_t n, const int32_t* src, const int32_t* dst,
+                                     const float* w, int64_t m_in, int32_t dup_policy,
+                                     int64_t* row_ptr, int32_t* col, float* val, float* deg,
+                                     int32_t* csr_eid, int32_t* eu, int32_t* ev, float* ew,
+                                     int64_t* m_out, void* ws, size_t ws_bytes, cudaStream_t s,
+                                     int* nonunit) {
   ERC_REQUIRE(n >= 1, "n must be >= 1 (got %d)", n);
   ERC_REQUIRE(m_in >= 0 && m_in <= (int64_t(1) << 30), "m_in out of range (%lld)",
               (long long)m_in);
@@ -228,7 +232,7 @@ extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const i
       ERC_CUDA(cudaMemsetAsync(p.upper, 0, (size_t)E, cs));  // slots past nnz must not count
       k_emit_csr<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, p.vals, p.head, p.slot, w, E, B,
                                                 dup_policy == ERC_DUP_FIRST, col, p.wmerged,
-                                                p.row_of, p.upper);
+                                                p.row_of, p.upper, w ? nullptr : p.err + 1);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
       k_row_ptr<<<grid_for(E, BT), BT, 0, cs>>>(p.row_of, p.counters, n, row_ptr);
@@ -256,15 +260,27 @@ extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const i
   key.add(row_ptr).add(col).add(val).add(deg).add(csr_eid).add(eu).add(ev).add(ew).add(a.base);
   ERC_TRY(graph_launch(key, enqueue, s));
   int64_t h_counters[2] = {0, 0};
-  unsigned h_err = 0;
+  unsigned h_err[2] = {0, 0};
   ERC_CUDA(cudaMemcpyAsync(h_counters, p.counters, 2 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
-  ERC_CUDA(cudaMemcpyAsync(&h_err, p.err, sizeof(unsigned), cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(h_err, p.err, 2 * sizeof(unsigned), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
-  if (h_err & 1u) return set_error(ERC_ERR_INVALID_ARG, "node id outside [0, %d)", n);
-  if (h_err & 2u) return set_error(ERC_ERR_INVALID_ARG, "edge weight not finite and positive");
+  if (h_err[0] & 1u) return set_error(ERC_ERR_INVALID_ARG, "node id outside [0, %d)", n);
+  if (h_err[0] & 2u) return set_error(ERC_ERR_INVALID_ARG, "edge weight not finite and positive");
   if (h_counters[0] != 2 * h_counters[1])
     return set_error(ERC_ERR_CUDA, "internal: nnz %lld != 2 m %lld", (long long)h_counters[0],
                      (long long)h_counters[1]);
   *m_out = h_counters[1];
+  if (nonunit) *nonunit = w ? 1 : (int)h_err[1];
   return ERC_OK;
+}
+
+extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const int32_t* dst,
+                                          const float* w, int64_t m_in, int32_t dup_policy,
+                                          int64_t* row_ptr, int32_t* col, float* val, float* deg,
+                                          int32_t* csr_eid, int32_t* eu, int32_t* ev, float* ew,
+                                          int64_t* m_out, void* ws, size_t ws_bytes,
+                                          erc_stream stream) {
+  clear_error();
+  return build_laplacian_impl(n, src, dst, w, m_in, dup_policy, row_ptr, col, val, deg, csr_eid,
+                              eu, ev, ew, m_out, ws, ws_bytes, as_stream(stream), nullptr);
 }

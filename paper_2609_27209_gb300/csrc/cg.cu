@@ -1836,10 +1836,10 @@ extern "C" size_t erc_batched_cg_workspace_size(int32_t n, int32_t ld) {
   return a.used + 256;
 }
 
-static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y, float* X,
-                                  int32_t ld, int32_t kc, float tol, int32_t max_iter,
-                                  int32_t* iters, float* relres, void* ws, size_t ws_bytes,
-                                  erc_stream stream, float* solve_us, int32_t* path) {
+erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float* X, int32_t ld,
+                           int32_t kc, float tol, int32_t max_iter, int32_t* iters, float* relres,
+                           void* ws, size_t ws_bytes, cudaStream_t s, bool reset_flags,
+                           cudaEvent_t ev0, cudaEvent_t ev1, int32_t* path) {
   ERC_TRY(check_graph(g));
   ERC_REQUIRE(kc >= 1 && ld >= kc && ld % 4 == 0 && ld <= MAX_LD, "bad kc %d / ld %d", kc, ld);
   ERC_REQUIRE(eps > 0.f && isfinite(eps), "eps must be positive");
@@ -1850,12 +1850,11 @@ static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y,
   ERC_TRY(check_block(X, "X"));
   if (ws_bytes < erc_batched_cg_workspace_size(g->n, ld))
     return set_error(ERC_ERR_CAPACITY, "workspace too small");
-  cudaStream_t s = as_stream(stream);
   Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
   CgWork w;
   plan_cg(ar, w, g->n, ld);
   ERC_CUDA(cudaMemsetAsync(w.cr.cnt, 0, colreduce_counter_bytes(), s));
-  ERC_CUDA(cudaMemsetAsync(w.flags, 0, 8 * sizeof(int), s));
+  if (reset_flags) ERC_CUDA(cudaMemsetAsync(w.flags, 0, 8 * sizeof(int), s));
   ERC_CUDA(cudaMemsetAsync(w.gen, 0, 8 * sizeof(unsigned), s));
 
   int sgrid = 1;
@@ -1934,12 +1933,7 @@ static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y,
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
-  cudaEvent_t ev[2] = {nullptr, nullptr};
-  if (solve_us) {
-    ERC_CUDA(cudaEventCreate(&ev[0]));
-    ERC_CUDA(cudaEventCreate(&ev[1]));
-    ERC_CUDA(cudaEventRecord(ev[0], s));
-  }
+  if (ev0) ERC_CUDA(cudaEventRecord(ev0, s));
   if (cluster) {
     ClusterArgs ca{};
     ca.row_ptr = g->row_ptr;
@@ -1980,29 +1974,55 @@ static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y,
       if (!h_any) break;
     }
   }
-  if (solve_us) ERC_CUDA(cudaEventRecord(ev[1], s));
+  if (ev1) ERC_CUDA(cudaEventRecord(ev1, s));
 
   // true residual of the returned iterate, plus the per-column outputs
   SpmmArgs ra = sa;
   ra.P = X;
   ERC_TRY(launch_spmm<MODE_RESID>(ra, sgrid, s));
+  return ERC_OK;
+}
+
+erc_status erc::cg_status(int32_t n, int32_t ld, int32_t columns, int32_t max_iter, void* ws,
+                          cudaStream_t s) {
+  Arena ar(reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255)));
+  CgWork w;
+  plan_cg(ar, w, n, ld);
   int h_flags[4] = {0, 0, 0, 0};
   ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 4 * sizeof(int), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
+  if (h_flags[3]) return set_error(ERC_ERR_TIMEOUT, "a bounded grid-wide wait timed out");
+  if (h_flags[1]) return set_error(ERC_ERR_NUMERIC, "non-finite or non-positive CG scalar");
+  if (h_flags[2])
+    return set_error(ERC_ERR_NOT_CONVERGED, "%d of %d columns reached max_iter=%d", h_flags[2],
+                     columns, max_iter);
+  return ERC_OK;
+}
+
+static erc_status batched_cg_impl(const erc_graph* g, float eps, const float* Y, float* X,
+                                  int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                  int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                  erc_stream stream, float* solve_us, int32_t* path) {
+  cudaStream_t s = as_stream(stream);
+  cudaEvent_t ev[2] = {nullptr, nullptr};
+  if (solve_us) {
+    ERC_CUDA(cudaEventCreate(&ev[0]));
+    ERC_CUDA(cudaEventCreate(&ev[1]));
+  }
+  erc_status st = cg_enqueue(g, eps, Y, X, ld, kc, tol, max_iter, iters, relres, ws, ws_bytes, s,
+                             true, ev[0], ev[1], path);
+  if (st == ERC_OK) st = cg_status(g->n, ld, kc, max_iter, ws, s);
   if (solve_us) {
     float ms = 0.f;
-    const cudaError_t e = cudaEventElapsedTime(&ms, ev[0], ev[1]);
+    const cudaError_t e =
+        st == ERC_OK || st == ERC_ERR_NOT_CONVERGED ? cudaEventElapsedTime(&ms, ev[0], ev[1])
+                                                    : cudaSuccess;
     cudaEventDestroy(ev[0]);
     cudaEventDestroy(ev[1]);
     if (e != cudaSuccess) return set_error(ERC_ERR_CUDA, "event timing: %s", cudaGetErrorString(e));
     *solve_us = 1000.f * ms;
   }
-  if (h_flags[3]) return set_error(ERC_ERR_TIMEOUT, "update kernel grid barrier timed out");
-  if (h_flags[1]) return set_error(ERC_ERR_NUMERIC, "non-finite or non-positive CG scalar");
-  if (h_flags[2])
-    return set_error(ERC_ERR_NOT_CONVERGED, "%d of %d columns reached max_iter=%d", h_flags[2],
-                     kc, max_iter);
-  return ERC_OK;
+  return st;
 }
 
 extern "C" erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* X,
