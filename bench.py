@@ -218,9 +218,16 @@ def run_ours(args, world, rank, local_rank):
     w_d = None if w is None else torch.from_numpy(w).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB of L2
 
+    mem = None
     if world == 1:
         ws = erc.erc_run_workspace(n, m_in, prm, dev)
         out = erc._run_outputs(n, m_in, K, dev)
+        # the library allocates nothing: a step's device memory is its workspace, outputs, inputs
+        nbytes = lambda t: t.numel() * t.element_size()
+        mem = {"workspace": nbytes(ws),
+               "outputs": sum(nbytes(t) for t in out.values() if torch.is_tensor(t)),
+               "inputs": nbytes(src_d) + nbytes(dst_d) + (0 if w_d is None else nbytes(w_d))}
+        mem["total"] = sum(mem.values())
 
         def step():
             return erc.erc_run(n, src_d, dst_d, w_d, prm, ws=ws, out=out)
@@ -298,6 +305,7 @@ def run_ours(args, world, rank, local_rank):
     # reported under "spmm".
     roof = None
     spmm = None
+    cusparse = None
     if rank == 0:
         g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
         P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
@@ -309,6 +317,23 @@ def run_ours(args, world, rank, local_rank):
         spmm = {"kernel": "k_spmm (L_eps P + p.Ap)", "launch_us": t_spmm * 1e6,
                 "algorithmic_bytes": op_bytes, "achieved": op_bytes / t_spmm / 1e9,
                 "frac": op_bytes / t_spmm / 1e9 / peak, "traffic": spmm_traffic(args.config)}
+        # library comparison point (run only): cuSPARSE SpMM of the adjacency, A P, through
+        # torch's CSR x dense product, timed with events on the current stream
+        vals = g.val if not g.unit_weights else torch.ones(2 * g.m, device=dev)
+        A = torch.sparse_csr_tensor(g.row_ptr, g.col.long(), vals, size=(n, n))
+        for _ in range(3):
+            A @ P
+        ca, cb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ca.record()
+        for _ in range(args.spmm_reps):
+            A @ P
+        cb.record()
+        cb.synchronize()
+        t_cs = ca.elapsed_time(cb) / 1e3 / args.spmm_reps
+        cusparse = {"kernel": "cuSPARSE SpMM A P (torch sparse CSR @ dense), run only",
+                    "launch_us": t_cs * 1e6, "achieved": op_bytes / t_cs / 1e9,
+                    "frac": op_bytes / t_cs / 1e9 / peak}
+        del A
         erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)  # warm
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
         if path in (1, 2):
@@ -346,7 +371,8 @@ def run_ours(args, world, rank, local_rank):
                            "eps": wl.eps, "tol": wl.tol,
                            "l2": "flushed (256 MiB write) before every timed step",
                            "parallelism": f"projection columns over {world} rank(s)"},
-                "roofline": roof, "spmm": spmm, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "cpu_baseline": cpu,
+                "e2e": e2e, "gpu_launches": launches, "device_memory_bytes": mem,
                 "clocks": clocks,
                 "cg_iters": None if it is None else {"mean": float(it.mean()),
                                                      "max": float(it.max())}}
