@@ -306,6 +306,7 @@ def run_ours(args, world, rank, local_rank):
     roof = None
     spmm = None
     cusparse = None
+    sampler = None
     if rank == 0:
         g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
         P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
@@ -334,6 +335,22 @@ def run_ours(args, world, rank, local_rank):
                     "launch_us": t_cs * 1e6, "achieved": op_bytes / t_cs / 1e9,
                     "frac": op_bytes / t_cs / 1e9 / peak}
         del A
+        # the curvature-guided subgraph samplers on this run's probabilities (§3.2), one call
+        # each (node budget n/10, edge budget m/10); each call synchronises to return its sizes
+        if res.get("prob_node") is not None and res.get("prob_edge") is not None:
+            sampler = {"node_budget": max(1, n // 10), "edge_budget": max(1, g.m // 10)}
+            runs = [(erc.ERC_SAMPLE_NODES, "node", res["prob_node"], sampler["node_budget"]),
+                    (erc.ERC_SAMPLE_EDGES, "edge", res["prob_edge"], sampler["edge_budget"])]
+            for kind, key, prob, b in runs:
+                sws = erc._workspace(erc.lib().erc_sample_workspace_size(n, g.m, b), dev)
+                erc.erc_sample_subgraph(g, kind, prob, b, 1, ws=sws)
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                for r in range(5):
+                    nodes_s, edges_s = erc.erc_sample_subgraph(g, kind, prob, b, 1, b * r, ws=sws)
+                torch.cuda.synchronize()
+                sampler[key + "_subgraph_us"] = (time.perf_counter() - t0) / 5 * 1e6
+                sampler[key + "_subgraph_size"] = [int(nodes_s.numel()), int(edges_s.numel())]
         erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)  # warm
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
         if path in (1, 2):
@@ -371,7 +388,7 @@ def run_ours(args, world, rank, local_rank):
                            "eps": wl.eps, "tol": wl.tol,
                            "l2": "flushed (256 MiB write) before every timed step",
                            "parallelism": f"projection columns over {world} rank(s)"},
-                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "cpu_baseline": cpu,
+                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": sampler, "cpu_baseline": cpu,
                 "e2e": e2e, "gpu_launches": launches, "device_memory_bytes": mem,
                 "clocks": clocks,
                 "cg_iters": None if it is None else {"mean": float(it.mean()),

@@ -201,6 +201,47 @@ erc_status erc_sampling_probs_noalloc(const erc_graph* g, const float* kappa, fl
                                       float* prob_node, float* prob_edge, erc_stream s);
 
 /* ---------------------------------------------------------------------------------------------
+ * erc_sample_subgraph -- one curvature-guided subgraph (§3.2: sampling proportional to the node
+ * weights of Eq. 7 or the edge weights of Eq. 8; the paper's ERC-LG-sub(node) / (edge) samplers
+ * follow GraphSAINT).
+ *
+ * kind ERC_SAMPLE_NODES: `budget` draws with replacement over the n nodes with probabilities
+ *   prob [n] (prob_node of erc_sampling_probs); the subgraph is induced on the distinct drawn
+ *   nodes.
+ * kind ERC_SAMPLE_EDGES: `budget` draws over the m canonical edges with prob [m] (prob_edge); the
+ *   nodes are the drawn edges' endpoints and the edges are the subgraph induced on them
+ *   (induced != 0, GraphSAINT) or the distinct drawn edges (induced == 0).
+ * A draw is exact: weights W_i = round(prob_i * 2^40) (prob_i must lie in [0, 1]; entries below
+ *   2^-41 are never drawn), draw k takes x = (word0 << 32) | word1 of Philox4x32-10 with key
+ *   (seed lo, seed hi) and counter (k lo, k hi, 0x53414D50, kind), and picks the smallest i with
+ *   W_0 + .. + W_i > floor(x * sum(W) / 2^64).  Draws k = first_draw .. first_draw + budget - 1,
+ *   so consecutive calls with advancing first_draw continue one random stream.
+ * Out: nodes [capacity n] ascending distinct node ids, *n_out (host); edges [capacity m]
+ *   ascending canonical edge ids, *m_out (host).  Deterministic.
+ * Errors: INVALID_ARG for a probability outside [0, 1] or all weights rounding to zero;
+ *   CAPACITY if ws_bytes < erc_sample_workspace_size(n, m, budget).  Synchronises s.
+ * ------------------------------------------------------------------------------------------- */
+enum { ERC_SAMPLE_NODES = 0, ERC_SAMPLE_EDGES = 1 };
+size_t erc_sample_workspace_size(int32_t n, int64_t m, int64_t budget);
+erc_status erc_sample_subgraph(const erc_graph* g, int32_t kind, const float* prob,
+                               int64_t budget, uint64_t seed, int64_t first_draw, int32_t induced,
+                               int32_t* nodes, int32_t* n_out, int32_t* edges, int64_t* m_out,
+                               void* ws, size_t ws_bytes, erc_stream s);
+
+/* erc_saint_counts -- GraphSAINT's pre-sampling counts: node_count[v] += 1 for each of the n_s
+ * distinct ids in nodes, edge_count[e] += 1 for each of the m_s distinct ids in edges (device
+ * int32 arrays [n] and [m], accumulated over calls; the caller zeroes them first).
+ * erc_saint_norm -- from counts over N subgraphs: lambda[v] = node_count[v] / N (loss
+ * normalisation, [n]) and, for CSR slot j of row v holding edge e, alpha[j] =
+ * edge_count[e] / node_count[v] (aggregator normalisation of the message into v, [2m]; 0 where
+ * node_count[v] = 0), each a correctly rounded float32 quotient.  N in [1, 2^24). */
+erc_status erc_saint_counts(const erc_graph* g, const int32_t* nodes, int32_t n_s,
+                            const int32_t* edges, int64_t m_s, int32_t* node_count,
+                            int32_t* edge_count, erc_stream s);
+erc_status erc_saint_norm(const erc_graph* g, const int32_t* node_count, const int32_t* edge_count,
+                          int32_t N, float* lambda, float* alpha, erc_stream s);
+
+/* ---------------------------------------------------------------------------------------------
  * erc_laplacian_apply -- AP = L_eps P for an n x ld block (the CG operator of Eq. 5), and, when
  * pAp is not NULL, pAp[c] = sum_u P[u,c] AP[u,c] as float64 (device [kc]).  Exposed for testing
  * and benchmarking the operator alone.

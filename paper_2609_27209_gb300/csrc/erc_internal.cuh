@@ -137,6 +137,20 @@ __device__ __forceinline__ float2 df_from_double(double v) {
   const float hi = (float)v;
   return make_float2(hi, (float)(v - (double)hi));
 }
+// Philox4x32-10 block function (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64
+// multiplies, with the key bumped by the Weyl constants between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+    k.x += 0x9E3779B9u;
+    k.y += 0xBB67AE85u;
+  }
+  return c;
+}
+
 // (a.x + a.y) / (b.x + b.y) rounded to float, without float64 arithmetic: Dekker's pair division
 // (T. J. Dekker, "A floating-point technique for extending the available precision", 1971) with
 // one correction step.  q0 b.x is subtracted exactly by the fused multiply-add.

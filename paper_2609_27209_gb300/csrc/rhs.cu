@@ -9,20 +9,6 @@
 namespace erc {
 namespace {
 
-// Philox4x32-10 block function (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32->64
-// multiplies, with the key bumped by the Weyl constants between rounds.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
-    k.x += 0x9E3779B9u;
-    k.y += 0xBB67AE85u;
-  }
-  return c;
-}
-
 // Row u of Y: the LPR lanes of a group walk u's CSR slots LPR at a time.  Lane l generates the
 // Philox blocks of slot jb + l (one per 128-column block its group covers) and the slot's signed
 // coefficient; the slots are then applied in CSR order, each lane taking from the generating

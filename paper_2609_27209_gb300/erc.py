@@ -71,6 +71,13 @@ _SIGS = {
                                   _c_p]),
     "erc_sampling_probs_noalloc": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _f32, _c_p, _c_p,
                                           _c_p]),
+    "erc_sample_workspace_size": (_sz, [_i32, _i64, _i64]),
+    "erc_sample_subgraph": (_i32, [ctypes.POINTER(ErcGraphC), _i32, _c_p, _i64, _u64, _i64, _i32,
+                                   _c_p, ctypes.POINTER(_i32), _c_p, ctypes.POINTER(_i64), _c_p,
+                                   _sz, _c_p]),
+    "erc_saint_counts": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _i32, _c_p, _i64, _c_p, _c_p,
+                                _c_p]),
+    "erc_saint_norm": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _c_p, _i32, _c_p, _c_p, _c_p]),
     "erc_laplacian_apply_workspace_size": (_sz, [_i32, _i32]),
     "erc_laplacian_apply": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _c_p,
                                    _c_p, _sz, _c_p]),
@@ -262,6 +269,41 @@ def erc_sampling_probs(g, kappa, eta=1e-8):
     _check(lib().erc_sampling_probs(ctypes.byref(gc), _ptr(kappa), eta, _ptr(pn), _ptr(pe),
                                     _ptr(ws), ws.numel(), _stream()))
     return pn, pe
+
+
+ERC_SAMPLE_NODES, ERC_SAMPLE_EDGES = 0, 1
+
+
+def erc_sample_subgraph(g, kind, prob, budget, seed, first_draw=0, induced=True, ws=None):
+    """One curvature-guided subgraph (see include/erc.h): (nodes int32, edges int32) on device."""
+    dev = g.row_ptr.device
+    nodes = torch.empty(max(g.n, 1), dtype=torch.int32, device=dev)
+    edges = torch.empty(max(g.m, 1), dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = _workspace(lib().erc_sample_workspace_size(g.n, g.m, budget), dev)
+    n_s, m_s = _i32(0), _i64(0)
+    gc = g.c()
+    _check(lib().erc_sample_subgraph(ctypes.byref(gc), kind, _ptr(prob), budget, seed, first_draw,
+                                     int(bool(induced)), _ptr(nodes), ctypes.byref(n_s),
+                                     _ptr(edges), ctypes.byref(m_s), _ptr(ws), ws.numel(),
+                                     _stream()))
+    return nodes[:n_s.value], edges[:m_s.value]
+
+
+def erc_saint_counts(g, nodes, edges, node_count, edge_count):
+    gc = g.c()
+    _check(lib().erc_saint_counts(ctypes.byref(gc), _ptr(nodes), nodes.numel(), _ptr(edges),
+                                  edges.numel(), _ptr(node_count), _ptr(edge_count), _stream()))
+
+
+def erc_saint_norm(g, node_count, edge_count, N):
+    dev = g.row_ptr.device
+    lam = torch.empty(g.n, dtype=torch.float32, device=dev)
+    alpha = torch.empty(max(2 * g.m, 1), dtype=torch.float32, device=dev)[:2 * g.m]
+    gc = g.c()
+    _check(lib().erc_saint_norm(ctypes.byref(gc), _ptr(node_count), _ptr(edge_count), N,
+                                _ptr(lam), _ptr(alpha), _stream()))
+    return lam, alpha
 
 
 def erc_sampling_probs_noalloc(g, kappa, eta=1e-8, out=None):
