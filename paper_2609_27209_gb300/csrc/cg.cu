@@ -179,12 +179,13 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
 }
 
 // acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots
-// q = qb + gl + LPR v < qend.  L2ONLY loads p through L2 only: required where p is rewritten
+// q = qb + gl + LPR v < qend whose bit v of `on` is set (the others keep acc).  L2ONLY loads p through L2 only: required where p is rewritten
 // within the same launch.
 template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false>
 __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int qb,
                                              int qend, const float4 (&pu)[VPL], int64_t j0,
-                                             int64_t j1, float4 (&acc)[VPL]) {
+                                             int64_t j1, float4 (&acc)[VPL],
+                                             unsigned on = ~0u) {
   constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
   for (int64_t jb = j0; jb < j1; jb += LPR) {
     const int64_t jj = jb + gl;
@@ -213,7 +214,7 @@ __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned
         for (int v = 0; v < VPL; ++v) {
           const int q = qb + gl + LPR * v;
           const float* src = a.P + (size_t)cj[k] * a.ld + 4 * q;
-          pv[k][v] = (q < qend && t + k < cnt)
+          pv[k][v] = (q < qend && t + k < cnt && ((on >> v) & 1u))
                          ? (L2ONLY ? __ldcg(reinterpret_cast<const float4*>(src)) : ld_f4(src))
                          : pu[v];
         }
@@ -554,7 +555,8 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
 // ---------------------------------------------------------------------------- resident CG
 // When r and Ap of every row fit in the SMs' shared memory, one cooperative launch runs the whole
 // solve.  Block b owns rows [b rb, b rb + rb): their r and Ap live in its shared memory, x and p
-// in global memory (p is gathered by other blocks).  Per iteration:
+// in global memory (p is gathered by other blocks); where room is left (PS), the block's own rows
+// of p are kept in shared memory too, and global p is only written and gathered.  Per iteration:
 //   A  Ap = L_eps p on own rows (heavy rows by the whole block), p.Ap    -> reduce: alpha
 //   B  x += alpha p, r -= alpha Ap, r.r                                  -> reduce: beta, stop
 //   C  p = r + beta p                                                    -> barrier
@@ -602,7 +604,7 @@ __device__ __forceinline__ void res_wait(const unsigned* arr, unsigned target, i
   __syncthreads();
 }
 
-template <int LPR, int VPL, bool WEIGHTED>
+template <int LPR, int VPL, bool WEIGHTED, bool PS>
 __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   extern __shared__ __align__(16) float dsm[];
   const SpmmArgs& a = ra.s;
@@ -618,11 +620,16 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   const int nrows = (int)max((int64_t)0, min((int64_t)a.n, r0 + ra.rb) - r0);
   float* rs = dsm;                                     // [rb][ld]  r of own rows
   float* aps = rs + (size_t)ra.rb * ld;                // [rb][ld]  Ap of own rows
-  float* comb = aps + (size_t)ra.rb * ld;              // [GPB][ld] heavy-row slices
-  float2* sbuf = reinterpret_cast<float2*>(comb + (size_t)GPB * ld);  // [ld]
-  float2* scratch = sbuf + ld;                         // [PWARPS][PCH] = 2 * PT entries
+  float* ps = aps + (size_t)ra.rb * ld;                // [rb][ld]  p of own rows (PS only)
+  float2* sbuf = reinterpret_cast<float2*>(PS ? ps + (size_t)ra.rb * ld : ps);  // [ld]
+  // one region, used as the heavy-row slices [GPB][ld] during A and as the reduction scratch
+  // [PWARPS][PCH] = 2 * PT float pairs after it
+  float* comb = reinterpret_cast<float*>(sbuf + ld);
+  float2* scratch = sbuf + ld;
   float2* part_pap = a.cr.part1;                       // [G][ld] block partials of p.Ap
-  float2* part_rr = a.cr.part1 + (size_t)G * ld;       // [G][ld] block partials of r.r
+  // [G][ld] block partials of r.r, rounded to float: sums of squares lose at most 2^-24 of
+  // their total that way, and every block reads half the bytes
+  float* part_rr = reinterpret_cast<float*>(a.cr.part1 + (size_t)G * ld);
   unsigned* arrivals = va.gen;
   // per-column CG state, the same in every block
   __shared__ float2 s_rr[RMAXLD], s_yy[RMAXLD];  // float pairs
@@ -634,6 +641,8 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   for (int idx = threadIdx.x; idx < nrows * nvec; idx += PT) {
     const int i = idx / nvec, q = idx % nvec;
     reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = ldcg_f4(va.R + (size_t)(r0 + i) * ld + 4 * q);
+    if (PS)
+      reinterpret_cast<float4*>(ps + (size_t)i * ld)[q] = ldcg_f4(a.P + (size_t)(r0 + i) * ld + 4 * q);
   }
   int any = 0;
   for (int c = threadIdx.x; c < ld; c += PT) {
@@ -669,6 +678,17 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     if (*(volatile int*)&va.flags[3] != 0) break;
     // ---------------- A: Ap = L_eps p on own rows, p.Ap
     if (nsync) res_wait(arrivals, nsync * G, va.flags);  // every block's p is written
+    // this lane's float4 slots with an active column: converged columns are neither gathered
+    // nor updated (their alpha is 0)
+    unsigned on = 0;
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q < nvec) {
+        const int4 act = reinterpret_cast<const int4*>(s_active)[q];
+        if (act.x | act.y | act.z | act.w) on |= 1u << v;
+      }
+    }
 #pragma unroll
     for (int v = 0; v < VPL; ++v)
 #pragma unroll
@@ -682,10 +702,12 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
-        pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
+        pu[v] = q >= nvec || !((on >> v) & 1u) ? f4_zero()
+                : PS ? reinterpret_cast<const float4*>(ps + (size_t)(u - r0) * ld)[q]
+                     : ldcg_f4(a.P + (size_t)u * ld + 4 * q);
         acc[v] = f4_zero();
       }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, s0, s1, acc);
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, s0, s1, acc, on);
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
@@ -727,10 +749,12 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
-        pu[v] = q < nvec ? ldcg_f4(a.P + (size_t)u * ld + 4 * q) : f4_zero();
+        pu[v] = q >= nvec || !((on >> v) & 1u) ? f4_zero()
+                : PS ? reinterpret_cast<const float4*>(ps + (size_t)i * ld)[q]
+                     : ldcg_f4(a.P + (size_t)u * ld + 4 * q);
         acc[v] = f4_zero();
       }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, j0, j1, acc);
+      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, j0, j1, acc, on);
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int q = gl + LPR * v;
@@ -783,9 +807,9 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
 #pragma unroll
         for (int v = 0; v < VPL; ++v) {
           const int i = i0 + k * GPB, q = gl + LPR * v;
-          if (i < nrows && q < nvec) {
+          if (i < nrows && q < nvec && ((on >> v) & 1u)) {
             const size_t o = (size_t)(r0 + i) * ld + 4 * q;
-            p[k][v] = ldcg_f4(a.P + o);
+            p[k][v] = PS ? reinterpret_cast<const float4*>(ps + (size_t)i * ld)[q] : ldcg_f4(a.P + o);
             x[k][v] = *reinterpret_cast<const float4*>(va.X + o);
           }
         }
@@ -794,7 +818,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
 #pragma unroll
         for (int v = 0; v < VPL; ++v) {
           const int i = i0 + k * GPB, q = gl + LPR * v;
-          if (i >= nrows || q >= nvec) continue;
+          if (i >= nrows || q >= nvec || !((on >> v) & 1u)) continue;
           float4 xx = x[k][v], r = reinterpret_cast<const float4*>(rs + (size_t)i * ld)[q];
           const float4 pp = p[k][v], ap = reinterpret_cast<const float4*>(aps + (size_t)i * ld)[q];
           xx.x = fmaf(al[v].x, pp.x, xx.x);
@@ -814,10 +838,11 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         }
     }
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    for (int c = threadIdx.x; c < ld; c += PT) part_rr[(size_t)blockIdx.x * ld + c] = sbuf[c];
+    for (int c = threadIdx.x; c < ld; c += PT)
+      part_rr[(size_t)blockIdx.x * ld + c] = __fadd_rn(sbuf[c].x, sbuf[c].y);
     res_arrive(arrivals);
     res_wait(arrivals, ++nsync * G, va.flags);
-    colsum_rows(part_rr, G, ld, sbuf, scratch);
+    colsum_rows_f(part_rr, G, ld, sbuf, scratch);
     any = 0;
     for (int c = threadIdx.x; c < ld; c += PT) {
       float be = 0.f;
@@ -864,7 +889,8 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         for (int v = 0; v < VPL; ++v) {
           const int i = i0 + k * GPB, q = gl + LPR * v;
           if (i < nrows && (act[v].x | act[v].y | act[v].z | act[v].w))
-            p[k][v] = ldcg_f4(a.P + (size_t)(r0 + i) * ld + 4 * q);
+            p[k][v] = PS ? reinterpret_cast<const float4*>(ps + (size_t)i * ld)[q]
+                         : ldcg_f4(a.P + (size_t)(r0 + i) * ld + 4 * q);
         }
 #pragma unroll
       for (int k = 0; k < NU; ++k)
@@ -879,6 +905,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
           if (act[v].z) pp.z = fmaf(be[v].z, pp.z, r.z);
           if (act[v].w) pp.w = fmaf(be[v].w, pp.w, r.w);
           *reinterpret_cast<float4*>(const_cast<float*>(a.P) + (size_t)(r0 + i) * ld + 4 * q) = pp;
+          if (PS) reinterpret_cast<float4*>(ps + (size_t)i * ld)[q] = pp;
         }
     }
     res_arrive(arrivals);
@@ -1513,12 +1540,16 @@ erc_status launch_update(const VecArgs& va, int grid, cudaStream_t s) {
 // ---- resident path selection: the kernel for this shape, its shared memory, and whether it fits
 int resident_lpr(int nvec) { return nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32; }
 
-const void* resident_kernel(int nvec, bool weighted) {
+const void* resident_kernel(int nvec, bool weighted, bool ps) {
   const void* k = nullptr;
   auto pick = [&](auto lpr, auto vpl) {
     constexpr int LPR = decltype(lpr)::value, VPL = decltype(vpl)::value;
-    k = weighted ? (const void*)k_cg_resident<LPR, VPL, true>
-                 : (const void*)k_cg_resident<LPR, VPL, false>;
+    if (ps)
+      k = weighted ? (const void*)k_cg_resident<LPR, VPL, true, true>
+                   : (const void*)k_cg_resident<LPR, VPL, false, true>;
+    else
+      k = weighted ? (const void*)k_cg_resident<LPR, VPL, true, false>
+                   : (const void*)k_cg_resident<LPR, VPL, false, false>;
   };
   if (nvec <= 4) pick(ic<4>{}, ic<1>{});
   else if (nvec <= 8) pick(ic<8>{}, ic<1>{});
@@ -1560,25 +1591,34 @@ size_t open_smem(const void* k) {
   return lim;
 }
 
+// shared memory of the resident kernel: r, Ap (and p with PS) of `rows` rows, the column
+// partials, and the region shared by the heavy-row slices and the reduction scratch
+size_t resident_smem(int64_t rows, int ld, bool ps) {
+  const size_t gpb = PT / resident_lpr(ld / 4);
+  const size_t shared = std::max(gpb * (size_t)ld, 4 * (size_t)PT);
+  return 4 * ((ps ? 3 : 2) * (size_t)rows * ld + 2 * (size_t)ld + shared);
+}
+
 bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const void** kern) {
   const int nvec = ld / 4;
-  const void* k = resident_kernel(nvec, g->val != nullptr);
-  if (!k) return false;
-  const int lpr = resident_lpr(nvec);
   const int grid = sm_count();
   const int64_t rows = ((int64_t)g->n + grid - 1) / grid;
-  const size_t bytes = 4 * (2 * (size_t)rows * ld + (size_t)(PT / lpr) * ld + 2 * (size_t)ld +
-                            2 * (size_t)PWARPS * PCH);
-  if (bytes > open_smem(k)) return false;
-  int nb = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, PT, bytes) != cudaSuccess || nb < 1) {
-    cudaGetLastError();
-    return false;
+  for (int ps = 1; ps >= 0; --ps) {  // p in shared memory when it fits
+    const void* k = resident_kernel(nvec, g->val != nullptr, ps);
+    if (!k) return false;
+    const size_t bytes = resident_smem(rows, ld, ps);
+    if (bytes > open_smem(k)) continue;
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, PT, bytes) != cudaSuccess || nb < 1) {
+      cudaGetLastError();
+      continue;
+    }
+    *rb = (int32_t)rows;
+    *smem = bytes;
+    *kern = k;
+    return true;
   }
-  *rb = (int32_t)rows;
-  *smem = bytes;
-  *kern = k;
-  return true;
+  return false;
 }
 
 erc_status launch_resident(const void* kern, const ResArgs& ra, size_t smem, cudaStream_t s) {

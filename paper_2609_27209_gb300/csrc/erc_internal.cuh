@@ -308,6 +308,49 @@ __device__ __forceinline__ void colsum_rows(const float2* part, int G, int ld, f
   __syncthreads();
 }
 
+// colsum_rows for float partials (part: [G][ld] floats, ld a multiple of 4, ld <= 2 blockDim.x):
+// four columns per load, float-pair sums in a fixed order; tmp holds 2 * blockDim.x entries.  For partials that are sums of squares, whose
+// rounding to float costs at most 2^-24 of the total.
+__device__ __forceinline__ void colsum_rows_f(const float* part, int G, int ld, float2* res,
+                                              float2* tmp) {
+  const int bd = blockDim.x;
+  const int quads = ld >> 2;
+  constexpr int CHUNK = 20;
+  // segments of the rows, as many as the threads and tmp's 2 * blockDim.x entries allow
+  const int nseg = max(1, min(quads <= bd ? bd / quads : 1, (2 * bd) / ld));
+  const int per = (G + nseg - 1) / nseg;
+  for (int t = threadIdx.x; t < nseg * quads; t += bd) {
+    const int seg = t / quads, cq = t % quads;
+    const int k0 = seg * per, k1 = min(G, k0 + per);
+    float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                   make_float2(0.f, 0.f)};
+    for (int k = k0; k < k1; k += CHUNK) {
+      float4 v[CHUNK];
+#pragma unroll
+      for (int j = 0; j < CHUNK; ++j)
+        v[j] = k + j < k1
+                   ? __ldcg(reinterpret_cast<const float4*>(part + (size_t)(k + j) * ld) + cq)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int j = 0; j < CHUNK; ++j) {
+        a[0] = df_add(a[0], make_float2(v[j].x, 0.f));
+        a[1] = df_add(a[1], make_float2(v[j].y, 0.f));
+        a[2] = df_add(a[2], make_float2(v[j].z, 0.f));
+        a[3] = df_add(a[3], make_float2(v[j].w, 0.f));
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) tmp[seg * ld + 4 * cq + i] = a[i];
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < ld; c += bd) {
+    float2 acc = make_float2(0.f, 0.f);
+    for (int s = 0; s < nseg; ++s) acc = df_add(acc, tmp[s * ld + c]);
+    res[c] = acc;
+  }
+  __syncthreads();
+}
+
 // ------------------------------------------------------------------------------------------------
 // row-block shapes: a row of ld floats is nvec = ld/4 float4s, handled by a group of LPR lanes
 // with VPL float4s per lane (LPR * VPL >= nvec).

@@ -165,3 +165,25 @@ def test_pipeline_batches_sum_to_whole():
     full = erc.erc_run(n, to_dev(src), to_dev(dst), None,
                        erc.Params(K=64, kc=64, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED))
     np.testing.assert_allclose(host(R), host(full["R"]), rtol=1e-4)
+
+
+def test_resident_solver_without_p_in_shared_memory(monkeypatch):
+    """12,000 nodes x 256 columns: r and Ap of a block's rows fit in shared memory but p does not,
+    so the resident kernel gathers and updates p in global memory only."""
+    monkeypatch.setenv("ERC_CG_MODE", "resident")
+    n, src, dst, w = synth.random_connected(12000, 36000, seed=31, weighted=True)
+    g, ref = build_both(n, src, dst, w)
+    kc = 256
+    Y = erc.erc_jl_rhs(g, 9, 256, 0, kc)
+    X, iters, relres, st, _, path = erc.erc_batched_cg_timed(g, 1e-3, Y, kc, 1e-6)
+    assert st == erc.ERC_OK and path == 1
+    cols = np.arange(0, kc, 16)  # a column subset keeps the float64 oracle solve short
+    Yr = O.jl_rhs(ref, 9, 256, 0, kc)[:, cols]
+    Xr, itr, _, _ = O.batched_cg(ref, 1e-3, Yr, 1e-6)
+    Xs = torch.zeros(n, len(cols), device=dev())
+    Xs[:] = X[:, torch.as_tensor(cols, device=dev())]
+    Rg = torch.zeros(g.m, device=dev())
+    erc.erc_edge_resistance(g, Xs.contiguous(), len(cols), Rg)
+    _check_R(host(Rg), O.edge_resistance(ref, Xr))
+    assert np.all(np.abs(host(iters)[cols] - itr) <= 0.1 * itr + 2)
+    assert np.all(host(relres) <= 2e-6)
