@@ -49,42 +49,88 @@ __device__ __forceinline__ int64_t block_exclusive_scan(int64_t v, int64_t* bloc
   return r;
 }
 
-template <class Load>
-__global__ void __launch_bounds__(SCAN_THREADS) k_scan_reduce(Load in, int64_t n, int64_t* sums) {
-  const int64_t base = (int64_t)blockIdx.x * SCAN_TILE;
-  int64_t s = 0;
-#pragma unroll
-  for (int j = 0; j < SCAN_IPT; ++j) {
-    int64_t i = base + j * SCAN_THREADS + threadIdx.x;
-    if (i < n) s += in(i);
-  }
-  __shared__ int64_t tot;
-  block_exclusive_scan(s, &tot);
-  __syncthreads();
-  if (threadIdx.x == 0) sums[blockIdx.x] = tot;
-}
+// Single-pass exclusive scan with decoupled look-back (D. Merrill, M. Garland, "Single-pass
+// Parallel Prefix Scan with Decoupled Look-back", 2016).  Tiles are claimed in order through an
+// atomic ticket, so a tile only waits on tiles that have already started.  Each tile publishes
+// its aggregate, then its inclusive prefix, in one 64-bit status word (value << 2 | flag, flag 1
+// = aggregate, 2 = inclusive prefix); the tile's first warp walks back over its predecessors,
+// 32 at a time, until it meets an inclusive prefix.  Integer sums: the result does not depend on
+// the order in which tiles finish.  Inputs are non-negative and their total below 2^62.
+constexpr unsigned LOOKBACK_SPINS = 1u << 22;
 
 template <class Load>
 __global__ void __launch_bounds__(SCAN_THREADS)
-    k_scan_apply(Load in, int64_t n, const int64_t* offsets, int64_t* out, int64_t* total) {
+    k_scan_onepass(Load in, int64_t n, unsigned long long* status, unsigned* ticket, int64_t* out,
+                   int64_t* total, unsigned* timeout) {
   __shared__ int64_t tile[SCAN_TILE];
-  const int64_t base = (int64_t)blockIdx.x * SCAN_TILE;
+  __shared__ unsigned s_tile;
+  __shared__ int64_t s_prefix;
+  if (threadIdx.x == 0) s_tile = atomicAdd(ticket, 1u);
+  __syncthreads();
+  const int64_t t = s_tile;
+  const int64_t base = t * SCAN_TILE;
 #pragma unroll
   for (int j = 0; j < SCAN_IPT; ++j) {
-    int j2 = j * SCAN_THREADS + threadIdx.x;
-    int64_t i = base + j2;
+    const int j2 = j * SCAN_THREADS + threadIdx.x;
+    const int64_t i = base + j2;
     tile[j2] = i < n ? in(i) : 0;
   }
   __syncthreads();
   int64_t v[SCAN_IPT];
-  int64_t s = 0;
+  int64_t sum = 0;
 #pragma unroll
   for (int j = 0; j < SCAN_IPT; ++j) {
     v[j] = tile[threadIdx.x * SCAN_IPT + j];
-    s += v[j];
+    sum += v[j];
   }
-  __shared__ int64_t tot;
-  int64_t run = block_exclusive_scan(s, &tot) + (offsets ? offsets[blockIdx.x] : 0);
+  __shared__ int64_t agg;
+  const int64_t excl = block_exclusive_scan(sum, &agg);
+  volatile unsigned long long* st = status;
+  if (threadIdx.x < 32) {  // the first warp publishes and looks back
+    const int lane = threadIdx.x;
+    if (t == 0) {
+      if (lane == 0) {
+        st[0] = ((unsigned long long)agg << 2) | 2ull;
+        s_prefix = 0;
+      }
+    } else {
+      if (lane == 0) st[t] = ((unsigned long long)agg << 2) | 1ull;
+      int64_t prefix = 0;
+      int64_t j = t - 1;
+      bool done = false;
+      while (!done) {
+        // lanes read predecessors j, j-1, ..., j-31 (those that exist)
+        const int64_t q = j - lane;
+        unsigned long long w = 0;
+        if (q >= 0) {
+          unsigned spins = 0;
+          while (((w = st[q]) & 3ull) == 0ull) {
+            if (++spins > LOOKBACK_SPINS) {  // bounded: record it and take zero
+              atomicOr(timeout, 1u);
+              w = 2ull;
+              break;
+            }
+          }
+        } else {
+          w = 2ull;  // before tile 0: an inclusive prefix of 0
+        }
+        const unsigned incl = __ballot_sync(0xffffffffu, (w & 3ull) == 2ull);
+        const int stop = incl ? __ffs(incl) - 1 : 32;  // nearest inclusive prefix
+        int64_t part = lane <= stop ? (int64_t)(w >> 2) : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+        prefix += part;
+        done = incl != 0;
+        j -= 32;
+      }
+      if (lane == 0) {
+        st[t] = ((unsigned long long)(prefix + agg) << 2) | 2ull;
+        s_prefix = prefix;
+      }
+    }
+  }
+  __syncthreads();
+  int64_t run = excl + s_prefix;
 #pragma unroll
   for (int j = 0; j < SCAN_IPT; ++j) {
     tile[threadIdx.x * SCAN_IPT + j] = run;
@@ -93,16 +139,16 @@ __global__ void __launch_bounds__(SCAN_THREADS)
   __syncthreads();
 #pragma unroll
   for (int j = 0; j < SCAN_IPT; ++j) {
-    int j2 = j * SCAN_THREADS + threadIdx.x;
-    int64_t i = base + j2;
+    const int j2 = j * SCAN_THREADS + threadIdx.x;
+    const int64_t i = base + j2;
     if (i < n) out[i] = tile[j2];
   }
-  if (total && blockIdx.x == gridDim.x - 1 && threadIdx.x == 0)
-    *total = (offsets ? offsets[blockIdx.x] : 0) + tot;
+  if (total && base + SCAN_TILE >= n && threadIdx.x == 0) *total = s_prefix + agg;
 }
 
 inline int64_t scan_blocks(int64_t n) { return (n + SCAN_TILE - 1) / SCAN_TILE; }
 
+// tmp: [status: ntiles u64][ticket, timeout]
 template <class Load>
 erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* tmp,
                      cudaStream_t s) {
@@ -110,20 +156,12 @@ erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* 
     if (total) ERC_CUDA(cudaMemsetAsync(total, 0, sizeof(int64_t), s));
     return ERC_OK;
   }
-  int64_t nb = scan_blocks(n);
-  if (nb == 1) {
-    k_scan_apply<<<1, SCAN_THREADS, 0, s>>>(in, n, (const int64_t*)nullptr, out, total);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    return ERC_OK;
-  }
-  int64_t* sums = tmp;
-  int64_t* rest = tmp + ((nb + 31) & ~int64_t(31));
-  k_scan_reduce<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, sums);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-  ERC_TRY(scan_impl(LoadI64{sums}, nb, sums, (int64_t*)nullptr, rest, s));
-  k_scan_apply<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, sums, out, total);
+  const int64_t nb = scan_blocks(n);
+  unsigned long long* status = reinterpret_cast<unsigned long long*>(tmp);
+  unsigned* ticket = reinterpret_cast<unsigned*>(status + nb);
+  ERC_CUDA(cudaMemsetAsync(status, 0, (size_t)nb * sizeof(unsigned long long) + 8, s));
+  k_scan_onepass<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, status, ticket, out, total,
+                                                       ticket + 1);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
@@ -213,14 +251,7 @@ __global__ void __launch_bounds__(RS_THREADS)
 }  // namespace
 
 size_t scan_temp_bytes(int64_t n) {
-  size_t total = 0;
-  int64_t m = n;
-  while (m > SCAN_TILE) {
-    int64_t nb = scan_blocks(m);
-    total += (size_t)((nb + 31) & ~int64_t(31)) * sizeof(int64_t);
-    m = nb;
-  }
-  return total + 256;
+  return (size_t)(scan_blocks(n > 0 ? n : 1) + 1) * sizeof(unsigned long long) + 256;
 }
 
 erc_status exclusive_scan_i64(const int64_t* in, const uint8_t* flags, int64_t* out, int64_t n,
