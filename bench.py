@@ -355,7 +355,11 @@ def run_ours(args, world, rank, local_rank):
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
         if path in (1, 2):
             T = int(it_cg.max().item())
-            algo = T * (op_bytes + UPDATE_BYTES_PER_ELEM * n * kc)
+            # T iterations, plus the launch's own initialisation (read Y; write P, X) and, in the
+            # resident kernel, the true residual (one operator application on X, Y read)
+            algo = T * (op_bytes + UPDATE_BYTES_PER_ELEM * n * kc) + 12 * n * kc
+            if path == 1:
+                algo += op_bytes + 4 * n * kc
             ach = algo / (solve_us * 1e-6) / 1e9
             kname = "k_cg_cluster" if path == 2 else "k_cg_resident"
             roof = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",

@@ -179,13 +179,14 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
 }
 
 // acc += sum_{j in [j0, j1)} w_j (p_u - p_{col_j}) for this lane's float4 column slots
-// q = qb + gl + LPR v < qend whose bit v of `on` is set (the others keep acc).  L2ONLY loads p through L2 only: required where p is rewritten
+// q = qb + gl + LPR v < qend whose bit v of `on` is set (the others keep acc); p is the n x ld
+// block src_rows.  L2ONLY loads p through L2 only: required where p is rewritten
 // within the same launch.
 template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false>
-__device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned gm, int qb,
-                                             int qend, const float4 (&pu)[VPL], int64_t j0,
-                                             int64_t j1, float4 (&acc)[VPL],
-                                             unsigned on = ~0u) {
+__device__ __forceinline__ void gather_range(const SpmmArgs& a, const float* __restrict__ src_rows,
+                                             int gl, unsigned gm, int qb, int qend,
+                                             const float4 (&pu)[VPL], int64_t j0, int64_t j1,
+                                             float4 (&acc)[VPL], unsigned on = ~0u) {
   constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
   for (int64_t jb = j0; jb < j1; jb += LPR) {
     const int64_t jj = jb + gl;
@@ -213,7 +214,7 @@ __device__ __forceinline__ void gather_range(const SpmmArgs& a, int gl, unsigned
 #pragma unroll
         for (int v = 0; v < VPL; ++v) {
           const int q = qb + gl + LPR * v;
-          const float* src = a.P + (size_t)cj[k] * a.ld + 4 * q;
+          const float* src = src_rows + (size_t)cj[k] * a.ld + 4 * q;
           pv[k][v] = (q < qend && t + k < cnt && ((on >> v) & 1u))
                          ? (L2ONLY ? __ldcg(reinterpret_cast<const float4*>(src)) : ld_f4(src))
                          : pu[v];
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(Spm
     const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
     float4 pu[VPL], acc[VPL];
     load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
-    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, 0, nvec, pu, s0, s1, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, a.P, gl, gm, 0, nvec, pu, s0, s1, acc);
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
@@ -337,7 +338,7 @@ __global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(Spm
     if (j1 - j0 > a.H) continue;
     float4 pu[VPL], acc[VPL];
     load_row<LPR, VPL>(a, u, gl, nvec, pu, acc);
-    gather_range<LPR, VPL, WEIGHTED>(a, gl, gm, 0, nvec, pu, j0, j1, acc);
+    gather_range<LPR, VPL, WEIGHTED>(a, a.P, gl, gm, 0, nvec, pu, j0, j1, acc);
     finish_row<LPR, VPL, MODE>(a, u, gl, nvec, pu, acc, dot);
   }
   if (MODE == MODE_APPLY && a.pap_out == nullptr) return;
@@ -604,6 +605,114 @@ __device__ __forceinline__ void res_wait(const unsigned* arr, unsigned target, i
   __syncthreads();
 }
 
+// floats of the region shared by the heavy-row slices [GPB][ld] and the reduction scratch
+// [2 * PT float pairs] of the resident kernel
+__host__ __device__ constexpr size_t resident_shared_floats_for(int gpb, int ld) {
+  return (size_t)gpb * ld > 4 * (size_t)PT ? (size_t)gpb * ld : 4 * (size_t)PT;
+}
+__device__ __forceinline__ size_t resident_shared_floats(int ld) {
+  const int nvec = ld >> 2;
+  const int lpr = nvec <= 4 ? 4 : nvec <= 8 ? 8 : nvec <= 16 ? 16 : 32;
+  return resident_shared_floats_for(PT / lpr, ld);
+}
+
+// o = L_eps s on the block's rows, s = src_rows (n x ld; the block's own rows are read from `own`
+// when it is not null): o_u = eps s_u + sum_v w_uv (s_u - s_v).  The block's rows heavier than
+// a.H (the ascending local list hv[0..nh)) are split over all its groups and combined in group
+// order; the others take one group each.  emit(i, v, s_u, o_u) runs once per row i and valid
+// float4 slot v of the lane (for heavy rows in group 0).  Slots whose bit in `on` is clear are
+// neither loaded nor gathered (s_u = 0 there).
+template <int LPR, int VPL, bool WEIGHTED, class Emit>
+__device__ __forceinline__ void block_apply(const SpmmArgs& a, const float* src_rows,
+                                            const float* own, int64_t r0, int nrows,
+                                            const int* hv, int nh, float* comb, int gl, int gi,
+                                            unsigned gm, unsigned on, Emit&& emit) {
+  constexpr int GPB = PT / LPR;
+  const int ld = a.ld, nvec = ld >> 2;
+  auto own_row = [&](int i, int v) -> float4 {
+    const int q = gl + LPR * v;
+    if (q >= nvec || !((on >> v) & 1u)) return f4_zero();
+    return own ? reinterpret_cast<const float4*>(own + (size_t)i * ld)[q]
+               : ldcg_f4(src_rows + (size_t)(r0 + i) * ld + 4 * q);
+  };
+  for (int hh = 0; hh < nh; ++hh) {
+    const int i = hv[hh];
+    const int64_t u = r0 + i;
+    const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+    const int64_t per = (j1 - j0 + GPB - 1) / GPB;
+    const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
+    float4 pu[VPL], acc[VPL];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      pu[v] = own_row(i, v);
+      acc[v] = f4_zero();
+    }
+    gather_range<LPR, VPL, WEIGHTED, true>(a, src_rows, gl, gm, 0, nvec, pu, s0, s1, acc, on);
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q < nvec) reinterpret_cast<float4*>(comb + gi * ld)[q] = acc[v];
+    }
+    __syncthreads();
+    if (gi == 0) {
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int q = gl + LPR * v;
+        if (q >= nvec) continue;
+        float4 s = f4_zero();
+        for (int g = 0; g < GPB; ++g) {
+          const float4 c = reinterpret_cast<const float4*>(comb + g * ld)[q];
+          s.x += c.x;
+          s.y += c.y;
+          s.z += c.z;
+          s.w += c.w;
+        }
+        float4 o;
+        o.x = fmaf(a.eps, pu[v].x, s.x);
+        o.y = fmaf(a.eps, pu[v].y, s.y);
+        o.z = fmaf(a.eps, pu[v].z, s.z);
+        o.w = fmaf(a.eps, pu[v].w, s.w);
+        emit(i, v, pu[v], o);
+      }
+    }
+    __syncthreads();
+  }
+  for (int i = gi; i < nrows; i += GPB) {
+    const int64_t u = r0 + i;
+    const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
+    if (j1 - j0 > a.H) continue;
+    float4 pu[VPL], acc[VPL];
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      pu[v] = own_row(i, v);
+      acc[v] = f4_zero();
+    }
+    gather_range<LPR, VPL, WEIGHTED, true>(a, src_rows, gl, gm, 0, nvec, pu, j0, j1, acc, on);
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q >= nvec) continue;
+      float4 o;
+      o.x = fmaf(a.eps, pu[v].x, acc[v].x);
+      o.y = fmaf(a.eps, pu[v].y, acc[v].y);
+      o.z = fmaf(a.eps, pu[v].z, acc[v].z);
+      o.w = fmaf(a.eps, pu[v].w, acc[v].w);
+      emit(i, v, pu[v], o);
+    }
+  }
+}
+
+// the block's part of a grid-wide column sum: publish the block's partials (row blockIdx.x of
+// part), count in, wait for every block, then sum all blocks' rows in a fixed order into sbuf
+__device__ __forceinline__ void res_reduce(float2* part, int ld, const float2* bpart,
+                                           float2* sbuf, float2* scratch, unsigned* arrivals,
+                                           unsigned& nsync, int* flags) {
+  for (int c = threadIdx.x; c < ld; c += PT) part[(size_t)blockIdx.x * ld + c] = bpart[c];
+  res_arrive(arrivals);
+  res_wait(arrivals, ++nsync * gridDim.x, flags);
+  colsum_rows(part, gridDim.x, ld, sbuf, scratch);
+}
+
 template <int LPR, int VPL, bool WEIGHTED, bool PS>
 __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   extern __shared__ __align__(16) float dsm[];
@@ -613,6 +722,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   constexpr int NU = RU > VPL ? RU / VPL : 1;  // rows whose loads are in flight together
   const int gl = threadIdx.x & (LPR - 1);
   const int gi = threadIdx.x / LPR;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ld = a.ld, nvec = ld >> 2;
   const int G = gridDim.x;
   const unsigned gm = group_mask<LPR>();
@@ -622,62 +732,108 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   float* aps = rs + (size_t)ra.rb * ld;                // [rb][ld]  Ap of own rows
   float* ps = aps + (size_t)ra.rb * ld;                // [rb][ld]  p of own rows (PS only)
   float2* sbuf = reinterpret_cast<float2*>(PS ? ps + (size_t)ra.rb * ld : ps);  // [ld]
-  // one region, used as the heavy-row slices [GPB][ld] during A and as the reduction scratch
-  // [PWARPS][PCH] = 2 * PT float pairs after it
+  // one region, used as the heavy-row slices [GPB][ld] in the operator and as the reduction
+  // scratch [PWARPS][PCH] = 2 * PT float pairs after it; then the local heavy-row list [rb]
   float* comb = reinterpret_cast<float*>(sbuf + ld);
   float2* scratch = sbuf + ld;
-  float2* part_pap = a.cr.part1;                       // [G][ld] block partials of p.Ap
-  // [G][ld] block partials of r.r, rounded to float: sums of squares lose at most 2^-24 of
-  // their total that way, and every block reads half the bytes
+  int* hv = reinterpret_cast<int*>(comb + resident_shared_floats(ld));
+  // block partials, one region per reduction kind so that no block overwrites partials another
+  // block may still be summing: [G][ld] each
+  float2* part_pap = a.cr.part1;
+  // r.r rounded to float: sums of squares lose at most 2^-24 of their total that way, and every
+  // block reads half the bytes
   float* part_rr = reinterpret_cast<float*>(a.cr.part1 + (size_t)G * ld);
+  float2* part_init = a.cr.part1 + 2 * (size_t)G * ld;
+  float2* part_res = a.cr.part1 + 3 * (size_t)G * ld;
   unsigned* arrivals = va.gen;
   // per-column CG state, the same in every block
   __shared__ float2 s_rr[RMAXLD], s_yy[RMAXLD];  // float pairs
   __shared__ __align__(16) float s_alpha[RMAXLD], s_beta[RMAXLD];
   __shared__ __align__(16) int s_active[RMAXLD];
   __shared__ int s_iters[RMAXLD], s_conv[RMAXLD];
-  __shared__ int64_t s_h0, s_h1;
+  __shared__ int s_nh, s_wcnt[PWARPS];
 
-  for (int idx = threadIdx.x; idx < nrows * nvec; idx += PT) {
-    const int i = idx / nvec, q = idx % nvec;
-    reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = ldcg_f4(va.R + (size_t)(r0 + i) * ld + 4 * q);
-    if (PS)
-      reinterpret_cast<float4*>(ps + (size_t)i * ld)[q] = ldcg_f4(a.P + (size_t)(r0 + i) * ld + 4 * q);
+  // ---- the block's rows heavier than a.H, ascending
+  if (threadIdx.x == 0) s_nh = 0;
+  __syncthreads();
+  for (int base = 0; base < nrows; base += PT) {
+    const int i = base + threadIdx.x;
+    const bool heavy = i < nrows && a.row_ptr[r0 + i + 1] - a.row_ptr[r0 + i] > a.H;
+    const unsigned bal = __ballot_sync(0xffffffffu, heavy);
+    if (lane == 0) s_wcnt[warp] = __popc(bal);
+    __syncthreads();
+    int off = s_nh, tot = 0;
+    for (int w = 0; w < PWARPS; ++w) {
+      if (w < warp) off += s_wcnt[w];
+      tot += s_wcnt[w];
+    }
+    if (heavy) hv[off + __popc(bal & ((1u << lane) - 1u))] = i;
+    __syncthreads();
+    if (threadIdx.x == 0) s_nh += tot;
+    __syncthreads();
   }
+  const int nh = s_nh;
+
+  // ---- r = p = y (columns kc.. zero), x = 0; y.y -> the per-column state
+  float2 dot[VPL][4];
+#pragma unroll
+  for (int v = 0; v < VPL; ++v)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
+  for (int i = gi; i < nrows; i += GPB) {
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+      const int q = gl + LPR * v;
+      if (q >= nvec) continue;
+      const size_t o = (size_t)(r0 + i) * ld + 4 * q;
+      float4 y = ld_f4(a.Y + o);
+      const int cb = 4 * q;
+      if (cb + 0 >= a.kc) y.x = 0.f;
+      if (cb + 1 >= a.kc) y.y = 0.f;
+      if (cb + 2 >= a.kc) y.z = 0.f;
+      if (cb + 3 >= a.kc) y.w = 0.f;
+      reinterpret_cast<float4*>(rs + (size_t)i * ld)[q] = y;
+      if (PS) reinterpret_cast<float4*>(ps + (size_t)i * ld)[q] = y;
+      *reinterpret_cast<float4*>(const_cast<float*>(a.P) + o) = y;
+      *reinterpret_cast<float4*>(va.X + o) = f4_zero();
+      dot[v][0] = df_fma(dot[v][0], y.x, y.x);
+      dot[v][1] = df_fma(dot[v][1], y.y, y.y);
+      dot[v][2] = df_fma(dot[v][2], y.z, y.z);
+      dot[v][3] = df_fma(dot[v][3], y.w, y.w);
+    }
+  }
+  unsigned nsync = 0;
+  block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
+  res_reduce(part_init, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);  // also publishes p
   int any = 0;
   for (int c = threadIdx.x; c < ld; c += PT) {
-    s_rr[c] = df_from_double(__ldcg(va.rr + c));
-    s_yy[c] = df_from_double(__ldcg(va.yy + c));
+    const float2 v = sbuf[c];
+    const double vd = df_value(v);
+    int act = 0, cv = 1;
+    if (c < a.kc) {
+      if (!isfinite(vd)) {
+        cv = 0;
+        if (blockIdx.x == 0) atomicOr(&va.flags[1], 1);
+      } else if (vd > 0.0 && !(vd <= va.tol2 * vd)) {
+        act = 1;
+        cv = 0;
+      }
+    }
+    s_yy[c] = v;
+    s_rr[c] = v;
     s_alpha[c] = 0.f;
     s_beta[c] = 0.f;
-    s_active[c] = __ldcg(va.active + c);
-    s_iters[c] = __ldcg(va.iters + c);
-    s_conv[c] = __ldcg(va.conv + c);
-    any |= s_active[c];
-  }
-  if (threadIdx.x == 0) {  // this block's slice of the ascending heavy-row list
-    const int64_t nh = a.nheavy ? *a.nheavy : 0;
-    int64_t lo = 0, hi = nh;
-    while (lo < hi) {
-      const int64_t mid = (lo + hi) >> 1;
-      if (a.heavy[mid] < r0) lo = mid + 1; else hi = mid;
-    }
-    s_h0 = lo;
-    hi = nh;
-    while (lo < hi) {
-      const int64_t mid = (lo + hi) >> 1;
-      if (a.heavy[mid] < r0 + nrows) lo = mid + 1; else hi = mid;
-    }
-    s_h1 = lo;
+    s_active[c] = act;
+    s_iters[c] = 0;
+    s_conv[c] = cv;
+    any |= act;
   }
   any = __syncthreads_or(any);
 
-  unsigned nsync = 0;
-  float2 dot[VPL][4];
   while (any) {
     if (*(volatile int*)&va.flags[3] != 0) break;
     // ---------------- A: Ap = L_eps p on own rows, p.Ap
-    if (nsync) res_wait(arrivals, nsync * G, va.flags);  // every block's p is written
+    if (nsync > 1) res_wait(arrivals, nsync * G, va.flags);  // every block's p is written
     // this lane's float4 slots with an active column: converged columns are neither gathered
     // nor updated (their alpha is 0)
     unsigned on = 0;
@@ -693,89 +849,17 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     for (int v = 0; v < VPL; ++v)
 #pragma unroll
       for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
-    for (int64_t hh = s_h0; hh < s_h1; ++hh) {
-      const int64_t u = a.heavy[hh];
-      const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
-      const int64_t per = (j1 - j0 + GPB - 1) / GPB;
-      const int64_t s0 = min(j1, j0 + gi * per), s1 = min(j1, s0 + per);
-      float4 pu[VPL], acc[VPL];
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        pu[v] = q >= nvec || !((on >> v) & 1u) ? f4_zero()
-                : PS ? reinterpret_cast<const float4*>(ps + (size_t)(u - r0) * ld)[q]
-                     : ldcg_f4(a.P + (size_t)u * ld + 4 * q);
-        acc[v] = f4_zero();
-      }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, s0, s1, acc, on);
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        if (q < nvec) reinterpret_cast<float4*>(comb + gi * ld)[q] = acc[v];
-      }
-      __syncthreads();
-      if (gi == 0) {
-#pragma unroll
-        for (int v = 0; v < VPL; ++v) {
-          const int q = gl + LPR * v;
-          if (q >= nvec) continue;
-          float4 s = f4_zero();
-          for (int g = 0; g < GPB; ++g) {
-            const float4 c = reinterpret_cast<const float4*>(comb + g * ld)[q];
-            s.x += c.x;
-            s.y += c.y;
-            s.z += c.z;
-            s.w += c.w;
-          }
-          float4 o;
-          o.x = fmaf(a.eps, pu[v].x, s.x);
-          o.y = fmaf(a.eps, pu[v].y, s.y);
-          o.z = fmaf(a.eps, pu[v].z, s.z);
-          o.w = fmaf(a.eps, pu[v].w, s.w);
-          reinterpret_cast<float4*>(aps + (size_t)(u - r0) * ld)[q] = o;
-          dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
-          dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
-          dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
-          dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
-        }
-      }
-      __syncthreads();
-    }
-    for (int i = gi; i < nrows; i += GPB) {
-      const int64_t u = r0 + i;
-      const int64_t j0 = a.row_ptr[u], j1 = a.row_ptr[u + 1];
-      if (j1 - j0 > a.H) continue;
-      float4 pu[VPL], acc[VPL];
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        pu[v] = q >= nvec || !((on >> v) & 1u) ? f4_zero()
-                : PS ? reinterpret_cast<const float4*>(ps + (size_t)i * ld)[q]
-                     : ldcg_f4(a.P + (size_t)u * ld + 4 * q);
-        acc[v] = f4_zero();
-      }
-      gather_range<LPR, VPL, WEIGHTED, true>(a, gl, gm, 0, nvec, pu, j0, j1, acc, on);
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int q = gl + LPR * v;
-        if (q >= nvec) continue;
-        float4 o;
-        o.x = fmaf(a.eps, pu[v].x, acc[v].x);
-        o.y = fmaf(a.eps, pu[v].y, acc[v].y);
-        o.z = fmaf(a.eps, pu[v].z, acc[v].z);
-        o.w = fmaf(a.eps, pu[v].w, acc[v].w);
-        reinterpret_cast<float4*>(aps + (size_t)i * ld)[q] = o;
-        dot[v][0] = df_fma(dot[v][0], pu[v].x, o.x);
-        dot[v][1] = df_fma(dot[v][1], pu[v].y, o.y);
-        dot[v][2] = df_fma(dot[v][2], pu[v].z, o.z);
-        dot[v][3] = df_fma(dot[v][3], pu[v].w, o.w);
-      }
-    }
+    block_apply<LPR, VPL, WEIGHTED>(
+        a, a.P, PS ? ps : nullptr, r0, nrows, hv, nh, comb, gl, gi, gm, on,
+        [&](int i, int v, float4 pu, float4 o) {
+          reinterpret_cast<float4*>(aps + (size_t)i * ld)[gl + LPR * v] = o;
+          dot[v][0] = df_fma(dot[v][0], pu.x, o.x);
+          dot[v][1] = df_fma(dot[v][1], pu.y, o.y);
+          dot[v][2] = df_fma(dot[v][2], pu.z, o.z);
+          dot[v][3] = df_fma(dot[v][3], pu.w, o.w);
+        });
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    for (int c = threadIdx.x; c < ld; c += PT) part_pap[(size_t)blockIdx.x * ld + c] = sbuf[c];
-    res_arrive(arrivals);
-    res_wait(arrivals, ++nsync * G, va.flags);
-    colsum_rows(part_pap, G, ld, sbuf, scratch);
+    res_reduce(part_pap, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);
     for (int c = threadIdx.x; c < ld; c += PT) {
       const float2 v = sbuf[c];
       float al = 0.f;
@@ -911,13 +995,35 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     res_arrive(arrivals);
     ++nsync;
   }
-  // the per-column results, identical in every block
+
+  // ---- true residual y - L_eps x of the returned iterate (every block's x is final: the last
+  // reduction ordered its writes), relative to ||y||; iterations and the unconverged count
+#pragma unroll
+  for (int v = 0; v < VPL; ++v)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) dot[v][t] = make_float2(0.f, 0.f);
+  block_apply<LPR, VPL, WEIGHTED>(
+      a, va.X, nullptr, r0, nrows, hv, nh, comb, gl, gi, gm, ~0u,
+      [&](int i, int v, float4, float4 o) {
+        const int q = gl + LPR * v, cb = 4 * q;
+        const float4 y = ld_f4(a.Y + (size_t)(r0 + i) * ld + 4 * q);
+        const float rx = cb + 0 < a.kc ? y.x - o.x : 0.f;
+        const float ry = cb + 1 < a.kc ? y.y - o.y : 0.f;
+        const float rz = cb + 2 < a.kc ? y.z - o.z : 0.f;
+        const float rw = cb + 3 < a.kc ? y.w - o.w : 0.f;
+        dot[v][0] = df_fma(dot[v][0], rx, rx);
+        dot[v][1] = df_fma(dot[v][1], ry, ry);
+        dot[v][2] = df_fma(dot[v][2], rz, rz);
+        dot[v][3] = df_fma(dot[v][3], rw, rw);
+      });
+  block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
+  res_reduce(part_res, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);
   if (blockIdx.x == 0)
-    for (int c = threadIdx.x; c < ld; c += PT) {
-      va.rr[c] = df_value(s_rr[c]);
-      va.iters[c] = s_iters[c];
-      va.conv[c] = s_conv[c];
-      va.active[c] = s_active[c];
+    for (int c = threadIdx.x; c < a.kc; c += PT) {
+      const float q = s_yy[c].x > 0.f ? df_div(sbuf[c], s_yy[c]) : 0.f;
+      a.relres_out[c] = sqrtf(fmaxf(q, 0.f));
+      a.iters_out[c] = s_iters[c];
+      if (!s_conv[c]) atomicAdd(&va.flags[2], 1);
     }
 }
 
@@ -1592,11 +1698,11 @@ size_t open_smem(const void* k) {
 }
 
 // shared memory of the resident kernel: r, Ap (and p with PS) of `rows` rows, the column
-// partials, and the region shared by the heavy-row slices and the reduction scratch
+// partials, the region shared by the heavy-row slices and the reduction scratch, and the local
+// heavy-row list
 size_t resident_smem(int64_t rows, int ld, bool ps) {
-  const size_t gpb = PT / resident_lpr(ld / 4);
-  const size_t shared = std::max(gpb * (size_t)ld, 4 * (size_t)PT);
-  return 4 * ((ps ? 3 : 2) * (size_t)rows * ld + 2 * (size_t)ld + shared);
+  const size_t shared = resident_shared_floats_for(PT / resident_lpr(ld / 4), ld);
+  return 4 * ((ps ? 3 : 2) * (size_t)rows * ld + 2 * (size_t)ld + shared + (size_t)rows);
 }
 
 bool resident_plan(const erc_graph* g, int ld, int32_t* rb, size_t* smem, const void** kern) {
@@ -1900,7 +2006,6 @@ erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float*
   int sgrid = 1;
   int32_t H = 0;
   spmm_shape(g, ld, &sgrid, &H);
-  ERC_TRY(build_heavy(g, H, w.heavy, s));
   const int nvec = ld / 4;
   const int ugrid = update_grid(g->n, nvec);
 
@@ -1968,7 +2073,10 @@ erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float*
       cluster = false;
   }
   if (path) *path = cluster ? 2 : resident ? 1 : 0;
-  if (!cluster) {  // the cluster kernel initialises its own columns
+  // the resident kernel finds its own heavy rows, initialises its columns and forms the true
+  // residual itself; the cluster kernel initialises its own columns
+  if (!resident) ERC_TRY(build_heavy(g, H, w.heavy, s));
+  if (!cluster && !resident) {
     k_cg_init<<<grid_for(g->n, vec_threads(nvec) / nvec), vec_threads(nvec), 0, s>>>(va);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
@@ -2017,9 +2125,11 @@ erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float*
   if (ev1) ERC_CUDA(cudaEventRecord(ev1, s));
 
   // true residual of the returned iterate, plus the per-column outputs
-  SpmmArgs ra = sa;
-  ra.P = X;
-  ERC_TRY(launch_spmm<MODE_RESID>(ra, sgrid, s));
+  if (!resident) {
+    SpmmArgs ra = sa;
+    ra.P = X;
+    ERC_TRY(launch_spmm<MODE_RESID>(ra, sgrid, s));
+  }
   return ERC_OK;
 }
 
