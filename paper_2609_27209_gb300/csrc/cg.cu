@@ -182,12 +182,12 @@ __device__ __forceinline__ void block_partials_rowgroup(float2 (&d)[VPL][4], flo
 // q = qb + gl + LPR v < qend whose bit v of `on` is set (the others keep acc); p is the n x ld
 // block src_rows.  L2ONLY loads p through L2 only: required where p is rewritten
 // within the same launch.
-template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false>
+template <int LPR, int VPL, bool WEIGHTED, bool L2ONLY = false, int UB = 8>
 __device__ __forceinline__ void gather_range(const SpmmArgs& a, const float* __restrict__ src_rows,
                                              int gl, unsigned gm, int qb, int qend,
                                              const float4 (&pu)[VPL], int64_t j0, int64_t j1,
                                              float4 (&acc)[VPL], unsigned on = ~0u) {
-  constexpr int U = VPL >= 8 ? 1 : 8 / VPL;  // neighbour rows in flight per group
+  constexpr int U = VPL >= UB ? 1 : UB / VPL;  // neighbour rows in flight per group
   for (int64_t jb = j0; jb < j1; jb += LPR) {
     const int64_t jj = jb + gl;
     int32_t cidx = 0;
@@ -574,6 +574,7 @@ constexpr int PWARPS = PT / 32;
 constexpr int PCH = 64;
 constexpr int RMAXLD = 256;  // widest row block the resident kernel takes (64 float4)
 constexpr int RU = 2;  // float4 loads per lane in flight in phases B and C
+constexpr int RUB = 8;  // neighbour rows in flight per row group in the gathers
 
 struct ResArgs {
   SpmmArgs s;
@@ -647,7 +648,7 @@ __device__ __forceinline__ void block_apply(const SpmmArgs& a, const float* src_
       pu[v] = own_row(i, v);
       acc[v] = f4_zero();
     }
-    gather_range<LPR, VPL, WEIGHTED, true>(a, src_rows, gl, gm, 0, nvec, pu, s0, s1, acc, on);
+    gather_range<LPR, VPL, WEIGHTED, true, RUB>(a, src_rows, gl, gm, 0, nvec, pu, s0, s1, acc, on);
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
@@ -687,7 +688,7 @@ __device__ __forceinline__ void block_apply(const SpmmArgs& a, const float* src_
       pu[v] = own_row(i, v);
       acc[v] = f4_zero();
     }
-    gather_range<LPR, VPL, WEIGHTED, true>(a, src_rows, gl, gm, 0, nvec, pu, j0, j1, acc, on);
+    gather_range<LPR, VPL, WEIGHTED, true, RUB>(a, src_rows, gl, gm, 0, nvec, pu, j0, j1, acc, on);
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
       const int q = gl + LPR * v;
