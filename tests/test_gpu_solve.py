@@ -81,18 +81,24 @@ def test_cg_paths_match_oracle(monkeypatch, mode, kc, weighted, heavy):
     assert np.all(host(relres) <= (4e-6 if heavy else 2e-6))
 
 
-def test_cg_not_converged_and_zero_columns():
+@pytest.mark.parametrize("mode", list(PATHS))
+def test_cg_not_converged_and_zero_columns(monkeypatch, mode):
+    monkeypatch.setenv("ERC_CG_MODE", mode)
     n, src, dst, w = synth.random_connected(1000, 3000, seed=5)
     g, ref = build_both(n, src, dst, w)
     Y = erc.erc_jl_rhs(g, 5, 16, 0, 16)
     Y[:, 3] = 0
-    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, 16, 1e-6, max_iter=3)
-    assert st == erc.ERC_ERR_NOT_CONVERGED
+    X, iters, relres, st, _, path = erc.erc_batched_cg_timed(g, 1e-3, Y, 16, 1e-6, max_iter=3)
+    assert st == erc.ERC_ERR_NOT_CONVERGED and path == PATHS[mode]
     it = host(iters)
     assert it[3] == 0 and np.all(np.delete(it, 3) == 3)
-    X, iters, relres, st = erc.erc_batched_cg(g, 1e-3, Y, 16, 1e-6)
+    X, iters, relres, st, _, path = erc.erc_batched_cg_timed(g, 1e-3, Y, 16, 1e-6)
     assert st == erc.ERC_OK and host(iters)[3] == 0 and float(host(relres)[3]) == 0.0
     assert torch.all(X[:, 3] == 0)
+    # a block whose every column is zero: nothing to iterate, the residual is zero
+    X, iters, relres, st, _, _ = erc.erc_batched_cg_timed(g, 1e-3, torch.zeros_like(Y), 16, 1e-6)
+    assert st == erc.ERC_OK and torch.all(iters == 0) and torch.all(relres == 0)
+    assert torch.all(X == 0)
 
 
 def test_cg_rejects_bad_arguments():
