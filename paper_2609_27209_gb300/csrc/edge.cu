@@ -131,7 +131,6 @@ struct ProbWork {
   double* part_qn;   // [MAX_GRID]
   double* part_cnt;  // [MAX_GRID]
   double* part_qe;   // [MAX_GRID]
-  double* scal;      // [0] kmin [1] kmax [2] sum qnode [3] #non-isolated [4] sum qedge
 };
 
 void plan_probs(Arena& a, ProbWork& w, int32_t n) {
@@ -141,7 +140,6 @@ void plan_probs(Arena& a, ProbWork& w, int32_t n) {
   w.part_qn = a.take<double>(MAX_GRID);
   w.part_cnt = a.take<double>(MAX_GRID);
   w.part_qe = a.take<double>(MAX_GRID);
-  w.scal = a.take<double>(8);
 }
 
 template <class V, class Op>
@@ -184,102 +182,97 @@ __global__ void __launch_bounds__(T)
   }
 }
 
-__global__ void __launch_bounds__(T) k_minmax_final(const float* part_min, const float* part_max,
-                                                    int nparts, double* scal) {
-  __shared__ float sh[T];
-  float lo = FLT_MAX, hi = -FLT_MAX;
-  for (int i = threadIdx.x; i < nparts; i += T) {
-    lo = fminf(lo, part_min[i]);
-    hi = fmaxf(hi, part_max[i]);
-  }
-  lo = block_reduce(lo, MinF{}, sh);
-  hi = block_reduce(hi, MaxF{}, sh);
-  if (threadIdx.x == 0) {
-    scal[0] = lo;
-    scal[1] = hi;
-  }
-}
-
-// Eq. 7 row sums: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta).
-// Each difference kappa - kappa_min is exact as a float pair; the row's pair sum is scaled once
-// in float64.  Per block: the sum of q_u and the number of non-isolated nodes.
-__global__ void __launch_bounds__(T)
-    k_qnode(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ eid,
-            const float* __restrict__ kappa, int32_t n, double eta, const double* scal,
-            double* __restrict__ qnode, double* part_qn, double* part_cnt) {
-  __shared__ double sh[T];
-  const int gl = threadIdx.x & (NL - 1);
-  const unsigned gm = group_mask<NL>();
-  const float kmin = (float)scal[0];  // the minimum of float kappa: exact
-  const double inv = 1.0 / (scal[1] - scal[0] + eta);
-  double tq = 0.0, tc = 0.0;
-  for (int64_t u = (int64_t)blockIdx.x * (T / NL) + threadIdx.x / NL; u < n;
-       u += (int64_t)gridDim.x * (T / NL)) {  // the same trip count for a group's lanes
-    const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
-    float2 acc = make_float2(0.f, 0.f);
-    for (int64_t j = j0 + gl; j < j1; j += NL)
-      acc = df_add(acc, df_two_sum(__ldg(kappa + __ldg(eid + j)), -kmin));
-    acc = group_df_sum(acc, gm);
-    if (gl == 0) {
-      const double q = df_value(acc) * inv;
-      qnode[u] = q;
-      tq += q;
-      tc += j1 > j0 ? 1.0 : 0.0;
-    }
-  }
-  tq = block_reduce(tq, AddD{}, sh);
-  tc = block_reduce(tc, AddD{}, sh);
-  if (threadIdx.x == 0) {
-    part_qn[blockIdx.x] = tq;
-    part_cnt[blockIdx.x] = tc;
-  }
-}
-
 // Eq. 8: q_e = sqrt(max(-kappa_e + 2 kappa_max, 0)) + 1
 __device__ __forceinline__ float edge_weight(float k, float kmax) {
   return sqrtf(fmaxf(-k + 2.f * kmax, 0.f)) + 1.f;
 }
 
-__global__ void __launch_bounds__(T)
-    k_qedge(const float* __restrict__ kappa, int64_t m, const double* scal, double* part_qe) {
-  __shared__ double sh[T];
-  const float kmax = (float)scal[1];
-  double acc = 0.0;
-  for (int64_t e = (int64_t)blockIdx.x * T + threadIdx.x; e < m; e += (int64_t)gridDim.x * T)
-    acc += (double)edge_weight(kappa[e], kmax);
-  acc = block_reduce(acc, AddD{}, sh);
-  if (threadIdx.x == 0) part_qe[blockIdx.x] = acc;
+// kappa_min and kappa_max from the blocks' partials of k_kappa_minmax, in the same order in every
+// block that needs them
+__device__ __forceinline__ void kappa_extrema(const float* part_min, const float* part_max,
+                                              int nparts, float* sh, float& kmin, float& kmax) {
+  float lo = FLT_MAX, hi = -FLT_MAX;
+  for (int i = threadIdx.x; i < nparts; i += T) {
+    lo = fminf(lo, part_min[i]);
+    hi = fmaxf(hi, part_max[i]);
+  }
+  kmin = block_reduce(lo, MinF{}, sh);
+  kmax = block_reduce(hi, MaxF{}, sh);
 }
 
-__global__ void __launch_bounds__(T) k_sums_final(const double* part_qn, const double* part_cnt,
-                                                  int np_node, const double* part_qe, int np_edge,
-                                                  double* scal) {
+// the Eq. 7 and Eq. 8 weights: blocks [0, gn) take node rows (q_u, per block the sum of q_u and
+// the number of non-isolated nodes), blocks [gn, gn + ge) take edges (per block the sum of q_e).
+// Node row sums: q_u = sum_{v in N(u)} (kappa_uv - kappa_min) / (kappa_max - kappa_min + eta);
+// each difference kappa - kappa_min is exact as a float pair, the row's pair sum is scaled once
+// in float64.
+__global__ void __launch_bounds__(T)
+    k_weights(const int64_t* __restrict__ row_ptr, const int32_t* __restrict__ eid,
+              const float* __restrict__ kappa, int32_t n, int64_t m, double eta,
+              const float* part_min, const float* part_max, int nmm, int gn,
+              double* __restrict__ qnode, double* part_qn, double* part_cnt, double* part_qe) {
+  __shared__ float shf[T];
   __shared__ double sh[T];
+  float kmin, kmax;
+  kappa_extrema(part_min, part_max, nmm, shf, kmin, kmax);
+  if ((int)blockIdx.x < gn) {
+    const int gl = threadIdx.x & (NL - 1);
+    const unsigned gm = group_mask<NL>();
+    const double inv = 1.0 / ((double)kmax - (double)kmin + eta);
+    double tq = 0.0, tc = 0.0;
+    for (int64_t u = (int64_t)blockIdx.x * (T / NL) + threadIdx.x / NL; u < n;
+         u += (int64_t)gn * (T / NL)) {  // the same trip count for a group's lanes
+      const int64_t j0 = row_ptr[u], j1 = row_ptr[u + 1];
+      float2 acc = make_float2(0.f, 0.f);
+      for (int64_t j = j0 + gl; j < j1; j += NL)
+        acc = df_add(acc, df_two_sum(__ldg(kappa + __ldg(eid + j)), -kmin));
+      acc = group_df_sum(acc, gm);
+      if (gl == 0) {
+        const double q = df_value(acc) * inv;
+        qnode[u] = q;
+        tq += q;
+        tc += j1 > j0 ? 1.0 : 0.0;
+      }
+    }
+    tq = block_reduce(tq, AddD{}, sh);
+    tc = block_reduce(tc, AddD{}, sh);
+    if (threadIdx.x == 0) {
+      part_qn[blockIdx.x] = tq;
+      part_cnt[blockIdx.x] = tc;
+    }
+  } else {
+    const int64_t b = (int64_t)blockIdx.x - gn, ge = (int64_t)gridDim.x - gn;
+    double acc = 0.0;
+    for (int64_t e = b * T + threadIdx.x; e < m; e += ge * T)
+      acc += (double)edge_weight(kappa[e], kmax);
+    acc = block_reduce(acc, AddD{}, sh);
+    if (threadIdx.x == 0) part_qe[b] = acc;
+  }
+}
+
+// normalisation: every block forms the three totals from all partials itself (same order in
+// every block), then scales its share of the node and edge weights
+__global__ void k_normalize(const int64_t* __restrict__ row_ptr, const double* __restrict__ qnode,
+                            int32_t n, const float* __restrict__ kappa, int64_t m,
+                            const float* part_min, const float* part_max, int nmm,
+                            const double* part_qn, const double* part_cnt, int gn,
+                            const double* part_qe, int ge, float* __restrict__ prob_node,
+                            float* __restrict__ prob_edge) {
+  __shared__ float shf[T];
+  __shared__ double sh[T];
+  float kmin, kmax;
+  kappa_extrema(part_min, part_max, nmm, shf, kmin, kmax);
   double a = 0.0, b = 0.0, c = 0.0;
-  for (int i = threadIdx.x; i < np_node; i += T) {
+  for (int i = threadIdx.x; i < gn; i += T) {
     a += part_qn[i];
     b += part_cnt[i];
   }
-  for (int i = threadIdx.x; i < np_edge; i += T) c += part_qe[i];
-  a = block_reduce(a, AddD{}, sh);
-  b = block_reduce(b, AddD{}, sh);
-  c = block_reduce(c, AddD{}, sh);
-  if (threadIdx.x == 0) {
-    scal[2] = a;
-    scal[3] = b;
-    scal[4] = c;
-  }
-}
-
-__global__ void k_normalize(const int64_t* __restrict__ row_ptr, const double* __restrict__ qnode,
-                            int32_t n, const float* __restrict__ kappa, int64_t m,
-                            const double* scal, float* __restrict__ prob_node,
-                            float* __restrict__ prob_edge) {
-  const double tot_n = scal[2], cnt = scal[3], tot_e = scal[4];
+  for (int i = threadIdx.x; i < ge; i += T) c += part_qe[i];
+  const double tot_n = block_reduce(a, AddD{}, sh);
+  const double cnt = block_reduce(b, AddD{}, sh);
+  const double tot_e = block_reduce(c, AddD{}, sh);
   const double inv_n = tot_n > 0.0 ? 1.0 / tot_n : 0.0;
   const double uni = cnt > 0.0 ? 1.0 / cnt : 0.0;
   const double inv_e = tot_e > 0.0 ? 1.0 / tot_e : 0.0;
-  const float kmax = (float)scal[1];
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n; u += stride) {
     double pr;
@@ -370,22 +363,16 @@ extern "C" erc_status erc_sampling_probs(const erc_graph* g, const float* kappa,
   k_kappa_minmax<<<ge, T, 0, s>>>(kappa, g->m, w.part_min, w.part_max);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
-  k_minmax_final<<<1, T, 0, s>>>(w.part_min, w.part_max, ge, w.scal);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
   const int gn = grid_for(g->n, T / NL);
-  k_qnode<<<gn, T, 0, s>>>(g->row_ptr, g->csr_eid, kappa, g->n, (double)eta, w.scal, w.qnode,
-                           w.part_qn, w.part_cnt);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-  k_qedge<<<ge, T, 0, s>>>(kappa, g->m, w.scal, w.part_qe);
-  count_launches(1);
-  ERC_CUDA(cudaGetLastError());
-  k_sums_final<<<1, T, 0, s>>>(w.part_qn, w.part_cnt, gn, w.part_qe, ge, w.scal);
+  const int gq = grid_for(g->m, T);  // edge blocks of the weights kernel (<= MAX_GRID partials)
+  k_weights<<<gn + gq, T, 0, s>>>(g->row_ptr, g->csr_eid, kappa, g->n, g->m, (double)eta,
+                                  w.part_min, w.part_max, ge, gn, w.qnode, w.part_qn, w.part_cnt,
+                                  w.part_qe);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   k_normalize<<<grid_for(g->n > g->m ? g->n : g->m, T), T, 0, s>>>(
-      g->row_ptr, w.qnode, g->n, kappa, g->m, w.scal, prob_node, prob_edge);
+      g->row_ptr, w.qnode, g->n, kappa, g->m, w.part_min, w.part_max, ge, w.part_qn,
+      w.part_cnt, gn, w.part_qe, gq, prob_node, prob_edge);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;

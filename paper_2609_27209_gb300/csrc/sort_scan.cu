@@ -168,41 +168,48 @@ erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* 
 }
 
 // ------------------------------------------------------------------------------------------------
-// radix sort: 8-bit digits, tiles of 2048 keys; a block's tile is split into 8 warp sub-tiles in
-// warp-striped order so that (warp, step, lane) order equals key order, which makes the ranks
-// stable.
+// radix sort: RB-bit digits (8, or 10 while the per-tile count table stays small: 3 passes instead
+// of 4 for the 30-bit keys of a 20k-node graph), tiles of 2048 keys; a block's tile is split into
+// 8 warp sub-tiles in warp-striped order so that (warp, step, lane) order equals key order, which
+// makes the ranks stable.
 // ------------------------------------------------------------------------------------------------
 constexpr int RS_THREADS = 256;
 constexpr int RS_WARPS = RS_THREADS / 32;
 constexpr int RS_IPT = 8;
 constexpr int RS_TILE = RS_THREADS * RS_IPT;
-constexpr int RS_RADIX = 256;
+constexpr int64_t RS_WIDE_MAX_TILES = 4096;  // 10-bit digits up to 8M keys
 
+inline int radix_bits(int64_t n) { return (n + RS_TILE - 1) / RS_TILE <= RS_WIDE_MAX_TILES ? 10 : 8; }
+
+template <int RB>
 __global__ void __launch_bounds__(RS_THREADS)
     k_radix_hist(const uint64_t* keys, int64_t n, int shift, int64_t* counts, int64_t nb) {
-  __shared__ unsigned hist[RS_RADIX];
-  for (int d = threadIdx.x; d < RS_RADIX; d += RS_THREADS) hist[d] = 0;
+  constexpr unsigned RADIX = 1u << RB;
+  __shared__ unsigned hist[RADIX];
+  for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS) hist[d] = 0;
   __syncthreads();
   const int64_t base = (int64_t)blockIdx.x * RS_TILE;
 #pragma unroll
   for (int j = 0; j < RS_IPT; ++j) {
     int64_t i = base + j * RS_THREADS + threadIdx.x;
-    if (i < n) atomicAdd(&hist[(unsigned)(keys[i] >> shift) & 255u], 1u);
+    if (i < n) atomicAdd(&hist[(unsigned)(keys[i] >> shift) & (RADIX - 1)], 1u);
   }
   __syncthreads();
-  for (int d = threadIdx.x; d < RS_RADIX; d += RS_THREADS)
+  for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS)
     counts[(int64_t)d * nb + blockIdx.x] = hist[d];
 }
 
+template <int RB>
 __global__ void __launch_bounds__(RS_THREADS)
     k_radix_scatter(const uint64_t* __restrict__ keys, const uint32_t* __restrict__ vals,
                     uint64_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n,
                     int shift, const int64_t* __restrict__ offsets, int64_t nb) {
-  __shared__ unsigned whist[RS_WARPS][RS_RADIX];
-  __shared__ int64_t boff[RS_RADIX];
+  constexpr unsigned RADIX = 1u << RB;
+  __shared__ unsigned whist[RS_WARPS][RADIX];
+  __shared__ int64_t boff[RADIX];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int d = threadIdx.x; d < RS_RADIX * RS_WARPS; d += RS_THREADS) (&whist[0][0])[d] = 0;
-  for (int d = threadIdx.x; d < RS_RADIX; d += RS_THREADS)
+  for (unsigned d = threadIdx.x; d < RADIX * RS_WARPS; d += RS_THREADS) (&whist[0][0])[d] = 0;
+  for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS)
     boff[d] = offsets[(int64_t)d * nb + blockIdx.x];
   __syncthreads();
   const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * 32 * RS_IPT;
@@ -217,7 +224,7 @@ __global__ void __launch_bounds__(RS_THREADS)
     bool ok = i < n;
     k[j] = ok ? keys[i] : 0;
     v[j] = ok ? vals[i] : 0;
-    unsigned d = ok ? ((unsigned)(k[j] >> shift) & 255u) : RS_RADIX;
+    unsigned d = ok ? ((unsigned)(k[j] >> shift) & (RADIX - 1)) : RADIX;
     dig[j] = d;
     unsigned peers = __match_any_sync(0xffffffffu, d);
     unsigned before = 0;
@@ -229,7 +236,7 @@ __global__ void __launch_bounds__(RS_THREADS)
   }
   __syncthreads();
   // exclusive prefix over warps per digit, plus the block's global offset for the digit
-  for (int d = threadIdx.x; d < RS_RADIX; d += RS_THREADS) {
+  for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS) {
     unsigned run = 0;
     for (int w = 0; w < RS_WARPS; ++w) {
       unsigned t = whist[w][d];
@@ -240,12 +247,42 @@ __global__ void __launch_bounds__(RS_THREADS)
   __syncthreads();
 #pragma unroll
   for (int j = 0; j < RS_IPT; ++j) {
-    if (dig[j] < RS_RADIX) {
+    if (dig[j] < RADIX) {
       int64_t dst = boff[dig[j]] + whist[warp][dig[j]] + rank[j];
       keys_out[dst] = k[j];
       vals_out[dst] = v[j];
     }
   }
+}
+
+template <int RB>
+erc_status radix_passes(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
+                        int64_t n, int bits, void* tmp, cudaStream_t s) {
+  const int64_t nb = (n + RS_TILE - 1) / RS_TILE;
+  const size_t cnt = (size_t)nb << RB;
+  char* t = static_cast<char*>(tmp);
+  int64_t* counts = reinterpret_cast<int64_t*>(t);
+  int64_t* offs = reinterpret_cast<int64_t*>(t + ((cnt * sizeof(int64_t) + 255) & ~size_t(255)));
+  void* scan_tmp = t + 2 * ((cnt * sizeof(int64_t) + 255) & ~size_t(255));
+  uint64_t *ka = keys, *kb = keys_alt;
+  uint32_t *va = vals, *vb = vals_alt;
+  int passes = 0;
+  for (int shift = 0; shift < bits; shift += RB, ++passes) {
+    k_radix_hist<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, n, shift, counts, nb);
+    count_launches(1);
+    ERC_CUDA(cudaGetLastError());
+    ERC_TRY(exclusive_scan_i64(counts, nullptr, offs, (int64_t)cnt, nullptr, scan_tmp, s));
+    k_radix_scatter<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, va, kb, vb, n, shift, offs, nb);
+    count_launches(1);
+    ERC_CUDA(cudaGetLastError());
+    uint64_t* tk = ka; ka = kb; kb = tk;
+    uint32_t* tv = va; va = vb; vb = tv;
+  }
+  if (passes & 1) {  // the result sits in the alternate buffers: copy it back
+    ERC_CUDA(cudaMemcpyAsync(keys, ka, (size_t)n * sizeof(uint64_t), cudaMemcpyDeviceToDevice, s));
+    ERC_CUDA(cudaMemcpyAsync(vals, va, (size_t)n * sizeof(uint32_t), cudaMemcpyDeviceToDevice, s));
+  }
+  return ERC_OK;
 }
 
 }  // namespace
@@ -261,39 +298,16 @@ erc_status exclusive_scan_i64(const int64_t* in, const uint8_t* flags, int64_t* 
 }
 
 size_t radix_sort_temp_bytes(int64_t n) {
-  int64_t nb = (n + RS_TILE - 1) / RS_TILE;
-  size_t cnt = (size_t)nb * RS_RADIX;
+  const int64_t nb = (n + RS_TILE - 1) / RS_TILE;
+  const size_t cnt = (size_t)nb << radix_bits(n);
   return 2 * ((cnt * sizeof(int64_t) + 255) & ~size_t(255)) + scan_temp_bytes((int64_t)cnt);
 }
 
 erc_status radix_sort_pairs(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
                             int64_t n, int bits, void* tmp, cudaStream_t s) {
   if (n <= 1) return ERC_OK;
-  int64_t nb = (n + RS_TILE - 1) / RS_TILE;
-  size_t cnt = (size_t)nb * RS_RADIX;
-  char* t = static_cast<char*>(tmp);
-  int64_t* counts = reinterpret_cast<int64_t*>(t);
-  int64_t* offs = reinterpret_cast<int64_t*>(t + ((cnt * sizeof(int64_t) + 255) & ~size_t(255)));
-  void* scan_tmp = t + 2 * ((cnt * sizeof(int64_t) + 255) & ~size_t(255));
-  uint64_t *ka = keys, *kb = keys_alt;
-  uint32_t *va = vals, *vb = vals_alt;
-  int passes = 0;
-  for (int shift = 0; shift < bits; shift += 8, ++passes) {
-    k_radix_hist<<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, n, shift, counts, nb);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    ERC_TRY(exclusive_scan_i64(counts, nullptr, offs, (int64_t)cnt, nullptr, scan_tmp, s));
-    k_radix_scatter<<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, va, kb, vb, n, shift, offs, nb);
-    count_launches(1);
-    ERC_CUDA(cudaGetLastError());
-    std::swap(ka, kb);
-    std::swap(va, vb);
-  }
-  if (passes & 1) {
-    ERC_CUDA(cudaMemcpyAsync(keys, ka, n * sizeof(uint64_t), cudaMemcpyDeviceToDevice, s));
-    ERC_CUDA(cudaMemcpyAsync(vals, va, n * sizeof(uint32_t), cudaMemcpyDeviceToDevice, s));
-  }
-  return ERC_OK;
+  if (radix_bits(n) == 10) return radix_passes<10>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s);
+  return radix_passes<8>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s);
 }
 
 }  // namespace erc
