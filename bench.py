@@ -167,6 +167,69 @@ def cpu_cores_used():
     return 1  # numpy elementwise and scipy sparse products run single-threaded here
 
 
+_THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+
+
+def _oracle_warm(_):
+    import numpy  # noqa: F401
+    import scipy.sparse  # noqa: F401
+
+    from oracle import erc_oracle  # noqa: F401
+    time.sleep(0.05)  # long enough that every worker of the pool takes a warm-up task
+    return os.getpid()
+
+
+def _oracle_columns(task):
+    """One worker's share of the oracle's column-proportional work (RHS, CG, distances)."""
+    name, K, c0, kc, g = task
+    from oracle import erc_oracle as O
+    from paper_2609_27209_gb300 import synth
+    wl = synth.WORKLOADS[name]
+    X, _, _, _ = O.batched_cg(g, wl.eps, O.jl_rhs(g, synth.JL_SEED, K, c0, kc), wl.tol)
+    return O.edge_resistance(g, X)
+
+
+def oracle_sample_all_cores(name, K, cols, procs):
+    """The same sample as oracle_sample with the `cols` columns split over `procs` processes
+    (spawn context, one BLAS thread each, warmed up before timing); the build and the
+    curvature/probability tail are not parallel and are timed once on one core."""
+    import multiprocessing as mp
+
+    from oracle import erc_oracle as O
+    from paper_2609_27209_gb300 import synth
+    n, src, dst, w = synth.make_graph(name)
+    t0 = time.perf_counter()
+    g = O.build_laplacian(n, src, dst, w)
+    t_build = time.perf_counter() - t0
+    saved = {k: os.environ.get(k) for k in _THREAD_VARS}
+    for k in _THREAD_VARS:
+        os.environ[k] = "1"
+    try:
+        with mp.get_context("spawn").Pool(procs) as pool:
+            pool.map(_oracle_warm, range(4 * procs), chunksize=1)
+            bounds = [(cols * i // procs, cols * (i + 1) // procs) for i in range(procs)]
+            tasks = [(name, K, a, b - a, g) for a, b in bounds if b > a]
+            t0 = time.perf_counter()
+            parts = pool.map(_oracle_columns, tasks, chunksize=1)
+            t_cols = time.perf_counter() - t0
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    R = sum(parts)
+    t0 = time.perf_counter()
+    _, kappa = O.curvature(g, R * (K / cols))
+    O.sampling_probs(g, kappa)
+    t_tail = time.perf_counter() - t0
+    est = t_build + t_cols * (K / cols) + t_tail
+    desc = (f"full graph (n={n}, m={g['m']}), {cols} of {K} projection columns split over "
+            f"{len(tasks)} processes; build and curvature/probability tail on one core, the "
+            f"column work scaled by {K}/{cols}")
+    return g["m"] / est, desc
+
+
 # ------------------------------------------------------------------------------------ main legs
 def run_reference(args, world, rank):
     from paper_2609_27209_gb300 import synth
@@ -307,6 +370,7 @@ def run_ours(args, world, rank, local_rank):
     spmm = None
     cusparse = None
     sampler = None
+    cpu_all = None
     if rank == 0:
         g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
         P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
@@ -380,6 +444,10 @@ def run_ours(args, world, rank, local_rank):
         per_col = est4 / K  # the probe's estimate is for all K columns
         cols = int(min(K, max(4, (15.0 / max(per_col, 1e-9)) // 4 * 4)))
         v, secs, desc, est = oracle_sample(args.config, K, cols)
+        procs = max(1, min(os.cpu_count() or 1, cols))
+        va, desc_all = oracle_sample_all_cores(args.config, K, cols, procs)
+        cpu_all = {"value": va, "unit": "edges/s", "cores": procs, "kind": "oracle",
+                   "sample": desc_all}
         cpu = {"value": v, "unit": "edges/s", "cores": cpu_cores_used(), "kind": "oracle",
                "sample": desc, "seconds": secs}
 
@@ -393,6 +461,7 @@ def run_ours(args, world, rank, local_rank):
                            "l2": "flushed (256 MiB write) before every timed step",
                            "parallelism": f"projection columns over {world} rank(s)"},
                 "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": sampler, "cpu_baseline": cpu,
+                "cpu_baseline_all_cores": cpu_all,
                 "e2e": e2e, "gpu_launches": launches, "device_memory_bytes": mem,
                 "clocks": clocks,
                 "cg_iters": None if it is None else {"mean": float(it.mean()),
