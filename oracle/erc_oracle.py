@@ -244,6 +244,46 @@ def batched_cg(g, eps, Y, tol, max_iter=20000):
     return X, iters, relres, not active.any()
 
 
+def batched_pcg(g, eps, Y, tol, max_iter=20000):
+    """Optional solver variant, not in the paper: column-wise Jacobi-preconditioned CG on
+    L_eps X = Y with M = diag(L_eps) = deg + eps (preconditioned CG as in Y. Saad, "Iterative
+    Methods for Sparse Linear Systems", Algorithm 9.1).  Same start (x = 0, r = y), same stop test
+    on the unpreconditioned recursive residual ||r|| <= tol ||y||, same outputs as batched_cg.
+    """
+    A = adjacency(g)
+    d = np.asarray(A.sum(axis=1)).ravel() + eps  # the diagonal of L_eps, float64
+    Y = np.asarray(Y, dtype=np.float64)
+    X = np.zeros_like(Y)
+    Rv = Y.copy()
+    Z = Rv / d[:, None]
+    P = Z.copy()
+    rz = np.einsum("ij,ij->j", Rv, Z)
+    yy = np.einsum("ij,ij->j", Y, Y)
+    active = yy > (tol * tol) * yy
+    iters = np.zeros(Y.shape[1], np.int64)
+    for _ in range(max_iter):
+        if not active.any():
+            break
+        AP = laplacian_matvec(g, eps, P, A)
+        pAp = np.einsum("ij,ij->j", P, AP)
+        alpha = np.where(active, rz / np.where(active, pAp, 1.0), 0.0)
+        X += alpha * P
+        Rv -= alpha * AP
+        rr = np.einsum("ij,ij->j", Rv, Rv)
+        Z = Rv / d[:, None]
+        rz_new = np.einsum("ij,ij->j", Rv, Z)
+        beta = np.where(active, rz_new / np.where(active, rz, 1.0), 0.0)
+        P = np.where(active, Z + beta * P, P)
+        rz = np.where(active, rz_new, rz)
+        iters += active
+        active = active & (rr > (tol * tol) * yy)
+    res = Y - laplacian_matvec(g, eps, X, A)
+    ny = np.sqrt(yy)
+    relres = np.where(ny > 0, np.sqrt(np.einsum("ij,ij->j", res, res)) / np.where(ny > 0, ny, 1),
+                      0.0)
+    return X, iters, relres, not active.any()
+
+
 # ------------------------------------------------------------------------------------------------
 # Eq. 6, Eq. 2: resistances on the original edges, then curvature
 # ------------------------------------------------------------------------------------------------
@@ -303,10 +343,11 @@ def sampling_probs(g, kappa, eta=1e-8):
 
 
 def erc_lg(n, src, dst, w, K, kc, eps, tol, seed, max_iter=20000, eta=1e-8, dup_policy="sum",
-           columns=None):
+           columns=None, precond=None):
     """Algorithm 1 on one device: stream the K columns in batches of kc, accumulate R, then Eq. 2
     and §3.2.  `columns` = (c0, c1) restricts the run to that column range (R then holds only
-    those columns' contributions)."""
+    those columns' contributions).  precond="jacobi" solves with batched_pcg instead of the
+    paper's CG."""
     g = build_laplacian(n, src, dst, w, dup_policy)
     c_lo, c_hi = (0, K) if columns is None else columns
     R = np.zeros(g["m"])
@@ -316,7 +357,8 @@ def erc_lg(n, src, dst, w, K, kc, eps, tol, seed, max_iter=20000, eta=1e-8, dup_
     for c0 in range(c_lo, c_hi, kc):
         k = min(kc, c_hi - c0)
         Y = jl_rhs(g, seed, K, c0, k)
-        X, it, rr, ok = batched_cg(g, eps, Y, tol, max_iter)
+        solve = batched_pcg if precond == "jacobi" else batched_cg
+        X, it, rr, ok = solve(g, eps, Y, tol, max_iter)
         R += edge_resistance(g, X)
         iters.append(it)
         relres.append(rr)

@@ -105,3 +105,40 @@ def test_rhs_rows_of_a_subgraph_with_global_edge_ids():
     ids = np.searchsorted(keys, sub["eu"].astype(np.int64) * n + sub["ev"])
     Ys = O.jl_rhs(sub, 7, 96, 32, 40, edge_ids=ids)
     np.testing.assert_allclose(Ys[S], Y[S], rtol=0, atol=1e-14)
+
+
+# ---- the optional Jacobi-preconditioned variant (not in the paper)
+
+@pytest.mark.parametrize("eps", [1e-3, 1e-1])
+def test_pcg_matches_direct_solve(eps):
+    g = _graph(4, n=150, extra=300)
+    Y = O.jl_rhs(g, 5, 32, 0, 32)
+    X, iters, relres, ok = O.batched_pcg(g, eps, Y, 1e-11)
+    assert ok
+    Z = D.jl_dense_solve(D.dense_laplacian(g["n"], g["eu"], g["ev"], g["ew"]), eps, Y)
+    np.testing.assert_allclose(X, Z, rtol=0, atol=1e-7 * np.abs(Z).max())
+    assert np.all(relres <= 1e-11 * 1.01)
+
+
+@pytest.mark.parametrize("graph", ["cycle", "complete"])
+def test_pcg_equals_cg_on_regular_graphs(graph):
+    """Every degree equal: M = cI, and preconditioned CG takes exactly CG's steps."""
+    n, src, dst, w = synth.cycle(200) if graph == "cycle" else synth.complete(40)
+    g = O.build_laplacian(n, src, dst, w)
+    Y = O.jl_rhs(g, 3, 16, 0, 16)
+    Xc, ic, _, _ = O.batched_cg(g, 1e-3, Y, 1e-9)
+    Xp, ip, _, _ = O.batched_pcg(g, 1e-3, Y, 1e-9)
+    np.testing.assert_array_equal(ip, ic)
+    np.testing.assert_allclose(Xp, Xc, rtol=1e-9, atol=1e-12 * np.abs(Xc).max())
+
+
+def test_pcg_needs_fewer_iterations_with_hubs():
+    """A 3,000-node Chung-Lu graph (degree exponent 2.2): degrees spread over orders of magnitude,
+    which Jacobi scaling removes (measured: 88 CG against 23 preconditioned iterations)."""
+    n, src, dst, w = synth.chung_lu(3000, 2.2, 20000, "unit", 7)
+    g = O.build_laplacian(n, src, dst, w)
+    Y = O.jl_rhs(g, 4, 8, 0, 8)
+    _, ic, _, okc = O.batched_cg(g, 1e-3, Y, 1e-6)
+    _, ip, rp, okp = O.batched_pcg(g, 1e-3, Y, 1e-6)
+    assert okc and okp and np.all(rp <= 1.01e-6)
+    assert ip.max() * 2 <= ic.max(), (ip.max(), ic.max())
