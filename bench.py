@@ -42,6 +42,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--spmm-reps", type=int, default=50)
+    ap.add_argument("--precond", choices=["none", "jacobi"], default="none",
+                    help="CG preconditioner of the whole step (the paper's method: none)")
     return ap.parse_args()
 
 
@@ -123,12 +125,19 @@ def _traffic(kernel, workload):
     if not os.path.exists(p):
         return None
     d = json.load(open(p))
-    src = os.path.join(ROOT, "paper_2609_27209_gb300", "csrc", "cg.cu")
-    sha = hashlib.sha1(open(src, "rb").read()).hexdigest()
     e = d.get(kernel, {}).get(workload)
-    if not e or e.get("cg_cu_sha1") != sha:
+    if not e or e.get("solver_src_sha1") != solver_src_sha1():
         return None
     return e.get("dram_bytes_per_launch")
+
+
+def solver_src_sha1():
+    """sha1 of the solver's sources (cg.cu, then cg_device.cuh): ncu counters taken on other
+    sources do not describe the kernels that run."""
+    h = hashlib.sha1()
+    for f in ("cg.cu", "cg_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2609_27209_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
 
 
 def spmm_algorithmic_bytes(n, m, kc, weighted):
@@ -137,7 +146,12 @@ def spmm_algorithmic_bytes(n, m, kc, weighted):
 
 
 # ------------------------------------------------------------------------------------ oracle leg
-def oracle_sample(name, K, cols):
+def _oracle_solver(precond):
+    from oracle import erc_oracle as O
+    return O.batched_pcg if precond == "jacobi" else O.batched_cg
+
+
+def oracle_sample(name, K, cols, precond="none"):
     """Time the CPU oracle on the full graph with `cols` of the K projection columns and
     extrapolate the column-proportional part to K.  Returns (edges/s, seconds, description)."""
     import numpy as np
@@ -151,7 +165,7 @@ def oracle_sample(name, K, cols):
     g = O.build_laplacian(n, src, dst, w)
     t1 = time.perf_counter()
     Y = O.jl_rhs(g, synth.JL_SEED, K, 0, cols)
-    X, it, _, _ = O.batched_cg(g, wl.eps, Y, wl.tol)
+    X, it, _, _ = _oracle_solver(precond)(g, wl.eps, Y, wl.tol)
     R = O.edge_resistance(g, X)
     t2 = time.perf_counter()
     p, kappa = O.curvature(g, R * (K / cols))
@@ -181,15 +195,16 @@ def _oracle_warm(_):
 
 def _oracle_columns(task):
     """One worker's share of the oracle's column-proportional work (RHS, CG, distances)."""
-    name, K, c0, kc, g = task
+    name, K, c0, kc, g, precond = task
     from oracle import erc_oracle as O
     from paper_2609_27209_gb300 import synth
     wl = synth.WORKLOADS[name]
-    X, _, _, _ = O.batched_cg(g, wl.eps, O.jl_rhs(g, synth.JL_SEED, K, c0, kc), wl.tol)
+    X, _, _, _ = _oracle_solver(precond)(g, wl.eps, O.jl_rhs(g, synth.JL_SEED, K, c0, kc),
+                                         wl.tol)
     return O.edge_resistance(g, X)
 
 
-def oracle_sample_all_cores(name, K, cols, procs):
+def oracle_sample_all_cores(name, K, cols, procs, precond="none"):
     """The same sample as oracle_sample with the `cols` columns split over `procs` processes
     (spawn context, one BLAS thread each, warmed up before timing); the build and the
     curvature/probability tail are not parallel and are timed once on one core."""
@@ -208,7 +223,7 @@ def oracle_sample_all_cores(name, K, cols, procs):
         with mp.get_context("spawn").Pool(procs) as pool:
             pool.map(_oracle_warm, range(4 * procs), chunksize=1)
             bounds = [(cols * i // procs, cols * (i + 1) // procs) for i in range(procs)]
-            tasks = [(name, K, a, b - a, g) for a, b in bounds if b > a]
+            tasks = [(name, K, a, b - a, g, precond) for a, b in bounds if b > a]
             t0 = time.perf_counter()
             parts = pool.map(_oracle_columns, tasks, chunksize=1)
             t_cols = time.perf_counter() - t0
@@ -240,10 +255,10 @@ def run_reference(args, world, rank):
     if rank != 0:
         return
     for _ in range(args.warmup):
-        oracle_sample(args.config, K, cols)
+        oracle_sample(args.config, K, cols, args.precond)
     vals, ests = [], []
     for _ in range(args.steps):
-        v, _, desc, est = oracle_sample(args.config, K, cols)
+        v, _, desc, est = oracle_sample(args.config, K, cols, args.precond)
         vals.append(v)
         ests.append(est)
     value = len(vals) / sum(1.0 / v for v in vals)  # harmonic mean = m / mean time
@@ -252,7 +267,7 @@ def run_reference(args, world, rank):
             "ms_per_step": 1000.0 * statistics.mean(ests), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": args.config, "K": K, "kc": wl.kc, "eps": wl.eps,
-                       "tol": wl.tol},
+                       "tol": wl.tol, "precond": args.precond},
             "cpu_baseline": {"value": value, "unit": "edges/s", "cores": cpu_cores_used(),
                              "kind": "oracle", "sample": desc},
             "e2e": {"value": value, "unit": "edges/s", "h2d_bytes_per_step": 0,
@@ -275,7 +290,9 @@ def run_ours(args, world, rank, local_rank):
     kc = min(wl.kc, K)
     n, src, dst, w = synth.make_graph(args.config)
     m_in = src.size
-    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
+    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED,
+                     precond=erc.ERC_PRECOND_JACOBI if args.precond == "jacobi"
+                     else erc.ERC_PRECOND_NONE)
     src_d = torch.from_numpy(src).to(dev)
     dst_d = torch.from_numpy(dst).to(dev)
     w_d = None if w is None else torch.from_numpy(w).to(dev)
@@ -371,6 +388,7 @@ def run_ours(args, world, rank, local_rank):
     cusparse = None
     sampler = None
     cpu_all = None
+    variants = None
     if rank == 0:
         g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
         P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
@@ -417,6 +435,19 @@ def run_ours(args, world, rank, local_rank):
                 sampler[key + "_subgraph_size"] = [int(nodes_s.numel()), int(edges_s.numel())]
         erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)  # warm
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
+        # the optional Jacobi-preconditioned solve of the same batch (not the paper's solver)
+        erc.erc_batched_pcg_timed(g, prm.eps, P, kc, prm.tol)
+        _, it_pc, _, _, pcg_us, pcg_path = erc.erc_batched_pcg_timed(g, prm.eps, P, kc, prm.tol)
+        variants = {"batch_columns": kc,
+                    "cg": {"path": path, "solve_us": solve_us,
+                           "iters_max": int(it_cg.max().item()),
+                           "iters_mean": float(it_cg.float().mean().item())},
+                    "jacobi_pcg": {"path": pcg_path, "solve_us": pcg_us,
+                                   "iters_max": int(it_pc.max().item()),
+                                   "iters_mean": float(it_pc.float().mean().item())}}
+        pc = args.precond == "jacobi"  # the roofline follows the solver the step runs
+        if pc:
+            it_cg, solve_us, path = it_pc, pcg_us, pcg_path
         if path in (1, 2):
             T = int(it_cg.max().item())
             # T iterations, plus the launch's own initialisation (read Y; write P, X) and, in the
@@ -427,8 +458,10 @@ def run_ours(args, world, rank, local_rank):
             ach = algo / (solve_us * 1e-6) / 1e9
             kname = "k_cg_cluster" if path == 2 else "k_cg_resident"
             roof = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
-                    "frac": ach / peak, "traffic": _traffic(kname[2:], args.config),
-                    "kernel": f"{kname} (one launch = whole CG solve of a batch)",
+                    "frac": ach / peak,
+                    "traffic": None if pc else _traffic(kname[2:], args.config),
+                    "kernel": f"{kname}{' (Jacobi)' if pc else ''} (one launch = whole CG solve "
+                              "of a batch)",
                     "iterations": T, "algorithmic_bytes": algo, "launch_us": solve_us,
                     "peak_source": src_kind}
         else:
@@ -440,12 +473,12 @@ def run_ours(args, world, rank, local_rank):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         # size the sample to roughly 15 s of CPU work from a 4-column probe
-        _, _, _, est4 = oracle_sample(args.config, K, 4)
+        _, _, _, est4 = oracle_sample(args.config, K, 4, args.precond)
         per_col = est4 / K  # the probe's estimate is for all K columns
         cols = int(min(K, max(4, (15.0 / max(per_col, 1e-9)) // 4 * 4)))
-        v, secs, desc, est = oracle_sample(args.config, K, cols)
+        v, secs, desc, est = oracle_sample(args.config, K, cols, args.precond)
         procs = max(1, min(os.cpu_count() or 1, cols))
-        va, desc_all = oracle_sample_all_cores(args.config, K, cols, procs)
+        va, desc_all = oracle_sample_all_cores(args.config, K, cols, procs, args.precond)
         cpu_all = {"value": va, "unit": "edges/s", "cores": procs, "kind": "oracle",
                    "sample": desc_all}
         cpu = {"value": v, "unit": "edges/s", "cores": cpu_cores_used(), "kind": "oracle",
@@ -457,10 +490,11 @@ def run_ours(args, world, rank, local_rank):
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
                 "config": {"workload": args.config, "n": n, "m": m, "K": K, "kc": kc,
-                           "eps": wl.eps, "tol": wl.tol,
+                           "eps": wl.eps, "tol": wl.tol, "precond": args.precond,
                            "l2": "flushed (256 MiB write) before every timed step",
                            "parallelism": f"projection columns over {world} rank(s)"},
-                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": sampler, "cpu_baseline": cpu,
+                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": sampler,
+                "solver_variants": variants, "cpu_baseline": cpu,
                 "cpu_baseline_all_cores": cpu_all,
                 "e2e": e2e, "gpu_launches": launches, "device_memory_bytes": mem,
                 "clocks": clocks,

@@ -48,6 +48,8 @@ typedef enum erc_status {
 } erc_status;
 
 enum { ERC_DUP_SUM = 0, ERC_DUP_FIRST = 1 };
+/* CG preconditioner: none (the paper's plain CG, the default) or Jacobi, M = diag(L_eps) */
+enum { ERC_PRECOND_NONE = 0, ERC_PRECOND_JACOBI = 1 };
 
 /* Non-owning view of a graph built by erc_build_laplacian (all pointers device, read-only). */
 typedef struct erc_graph {
@@ -73,6 +75,7 @@ typedef struct erc_params {
   int32_t max_iter;   /* CG iteration cap per column */
   float eta;          /* eta > 0 of Eq. 7 */
   int32_t dup_policy; /* ERC_DUP_SUM or ERC_DUP_FIRST */
+  int32_t precond;    /* ERC_PRECOND_NONE (Algorithm 1's plain CG) or ERC_PRECOND_JACOBI */
 } erc_params;
 
 const char* erc_version(void);
@@ -140,13 +143,29 @@ erc_status erc_batched_cg(const erc_graph* g, float eps, const float* Y, float* 
  *      (graphs whose rows' r and Ap slices fit in the shared memory of a cluster, when a cost
  *      model favours it over 1: small graphs); the launch also initialises r, p and x;
  *   1  one cooperative launch over all rows and columns (r and Ap blocks in the SMs' shared
- *      memory; separate initialisation kernel, not timed);
+ *      memory); the launch also initialises r, p and x and forms the true residual;
  *   0  the multi-kernel loop captured in CUDA graphs (larger graphs).
  * The environment variable ERC_CG_MODE=cluster|resident|graph restricts the choice. */
 erc_status erc_batched_cg_timed(const erc_graph* g, float eps, const float* Y, float* X,
                                 int32_t ld, int32_t kc, float tol, int32_t max_iter,
                                 int32_t* iters, float* relres, void* ws, size_t ws_bytes,
                                 float* solve_us, int32_t* path, erc_stream s);
+
+/* erc_batched_pcg, erc_batched_pcg_timed -- an optional solver variant, not part of the paper's
+ * method: erc_batched_cg with the Jacobi preconditioner M = diag(L_eps) = deg + eps (g->deg
+ * required), i.e. preconditioned CG (Y. Saad, "Iterative Methods for Sparse Linear Systems",
+ * Algorithm 9.1) with z = r / (deg + eps), p0 = z0, alpha = r.z / p.Ap, beta = r'.z' / r.z.
+ * Same arguments, workspace (erc_batched_cg_workspace_size), start (x = 0), stop test (on the
+ * unpreconditioned ||r||_2 <= tol ||y||_2), outputs and errors as erc_batched_cg.  It solves
+ * the same systems to the same tolerance in fewer iterations where degrees vary widely
+ * (power-law graphs).  Paths 1 and 0 only (no cluster solver). */
+erc_status erc_batched_pcg(const erc_graph* g, float eps, const float* Y, float* X, int32_t ld,
+                           int32_t kc, float tol, int32_t max_iter, int32_t* iters, float* relres,
+                           void* ws, size_t ws_bytes, erc_stream s);
+erc_status erc_batched_pcg_timed(const erc_graph* g, float eps, const float* Y, float* X,
+                                 int32_t ld, int32_t kc, float tol, int32_t max_iter,
+                                 int32_t* iters, float* relres, void* ws, size_t ws_bytes,
+                                 float* solve_us, int32_t* path, erc_stream s);
 
 /* ---------------------------------------------------------------------------------------------
  * erc_edge_resistance -- R_acc[e] += sum_{c < kc} (X[eu[e], c] - X[ev[e], c])^2   (Eq. 6).

@@ -217,7 +217,8 @@ erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, cons
     const int32_t k = prm->kc < prm->K - c0 ? prm->kc : prm->K - c0;
     ERC_TRY(erc_jl_rhs(&g, prm->seed, prm->K, c0, k, p.Y, ld, reinterpret_cast<erc_stream>(s)));
     ERC_TRY(cg_enqueue(&g, prm->eps, p.Y, p.X, ld, k, prm->tol, prm->max_iter, iters + c0,
-                       relres + c0, p.cg_ws, p.cg_bytes, s, c0 == 0, nullptr, nullptr, nullptr));
+                       relres + c0, p.cg_ws, p.cg_bytes, s, c0 == 0, nullptr, nullptr, nullptr,
+                       prm->precond == ERC_PRECOND_JACOBI));
     ERC_TRY(erc_edge_resistance(&g, p.X, ld, k, R, reinterpret_cast<erc_stream>(s)));
   }
   ERC_TRY(erc_curvature(&g, R, p_node, kappa, reinterpret_cast<erc_stream>(s)));
@@ -232,6 +233,8 @@ erc_status check_params(const erc_params* prm, int32_t n, int64_t m_in) {
   ERC_REQUIRE(prm->kc >= 1 && prm->kc <= MAX_LD, "kc must be in [1, %d]", MAX_LD);
   ERC_REQUIRE(prm->kc % 4 == 0 || prm->kc >= prm->K, "kc must be a multiple of 4 when K > kc");
   ERC_REQUIRE(n >= 1 && m_in >= 0, "bad n / m_in");
+  ERC_REQUIRE(prm->precond == ERC_PRECOND_NONE || prm->precond == ERC_PRECOND_JACOBI,
+              "precond must be ERC_PRECOND_NONE or ERC_PRECOND_JACOBI");
   return ERC_OK;
 }
 

@@ -75,9 +75,10 @@ erc_status graph_launch(GraphKey key, F&& enqueue, cudaStream_t s) {
 // Internal forms of the entry points for the whole-path driver.
 //   build_laplacian_impl: erc_build_laplacian, plus *nonunit (host, may be null) = 1 when some
 //     merged weight differs from 1 (always 1 for weighted input), read with m in one round trip.
-//   cg_enqueue: erc_batched_cg up to the true residual, without reading the status; the status
-//     flags accumulate over calls until reset_flags (the multi-kernel solver still polls its own
-//     progress).  cg_status reads them once: the status of every batch since the last reset.
+//   cg_enqueue: erc_batched_cg (erc_batched_pcg with precond) up to the true residual, without
+//     reading the status; the status flags accumulate over calls until reset_flags (the
+//     multi-kernel solver still polls its own progress).  cg_status reads them once: the status
+//     of every batch since the last reset.
 erc_status build_laplacian_impl(int32_t n, const int32_t* src, const int32_t* dst, const float* w,
                                 int64_t m_in, int32_t dup_policy, int64_t* row_ptr, int32_t* col,
                                 float* val, float* deg, int32_t* csr_eid, int32_t* eu, int32_t* ev,
@@ -86,7 +87,7 @@ erc_status build_laplacian_impl(int32_t n, const int32_t* src, const int32_t* ds
 erc_status cg_enqueue(const erc_graph* g, float eps, const float* Y, float* X, int32_t ld,
                       int32_t kc, float tol, int32_t max_iter, int32_t* iters, float* relres,
                       void* ws, size_t ws_bytes, cudaStream_t s, bool reset_flags,
-                      cudaEvent_t ev0, cudaEvent_t ev1, int32_t* path);
+                      cudaEvent_t ev0, cudaEvent_t ev1, int32_t* path, bool precond);
 erc_status cg_status(int32_t n, int32_t ld, int32_t columns, int32_t max_iter, void* ws,
                      cudaStream_t s);
 

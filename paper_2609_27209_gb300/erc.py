@@ -25,6 +25,8 @@ ERC_ERR_NUMERIC = 5
 ERC_ERR_TIMEOUT = 6
 ERC_DUP_SUM = 0
 ERC_DUP_FIRST = 1
+ERC_PRECOND_NONE = 0
+ERC_PRECOND_JACOBI = 1
 
 _c_p = ctypes.c_void_p
 _i32 = ctypes.c_int32
@@ -47,7 +49,7 @@ class ErcGraphC(ctypes.Structure):
 
 class ErcParamsC(ctypes.Structure):
     _fields_ = [("seed", _u64), ("K", _i32), ("kc", _i32), ("eps", _f32), ("tol", _f32),
-                ("max_iter", _i32), ("eta", _f32), ("dup_policy", _i32)]
+                ("max_iter", _i32), ("eta", _f32), ("dup_policy", _i32), ("precond", _i32)]
 
 
 _SIGS = {
@@ -64,6 +66,11 @@ _SIGS = {
     "erc_batched_cg_timed": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32,
                                     _f32, _i32, _c_p, _c_p, _c_p, _sz, ctypes.POINTER(_f32),
                                     ctypes.POINTER(_i32), _c_p]),
+    "erc_batched_pcg": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _f32,
+                               _i32, _c_p, _c_p, _c_p, _sz, _c_p]),
+    "erc_batched_pcg_timed": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32,
+                                     _f32, _i32, _c_p, _c_p, _c_p, _sz, ctypes.POINTER(_f32),
+                                     ctypes.POINTER(_i32), _c_p]),
     "erc_edge_resistance": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _i32, _i32, _c_p, _c_p]),
     "erc_curvature": (_i32, [ctypes.POINTER(ErcGraphC), _c_p, _c_p, _c_p, _c_p]),
     "erc_sampling_probs_workspace_size": (_sz, [_i32, _i64]),
@@ -208,8 +215,7 @@ def erc_jl_rhs(g, seed, K, c0, kc, ld=None, out=None):
     return Y
 
 
-def erc_batched_cg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
-    """Returns (X, iters, relres, status); status is ERC_OK or ERC_ERR_NOT_CONVERGED."""
+def _solve(fn, g, eps, Y, kc, tol, max_iter, X, ws, timed):
     n, ld = Y.shape
     dev = Y.device
     X = torch.empty_like(Y) if X is None else X
@@ -218,30 +224,37 @@ def erc_batched_cg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
     if ws is None:
         ws = _workspace(lib().erc_batched_cg_workspace_size(n, ld), dev)
     gc = g.c()
-    st = _check(lib().erc_batched_cg(ctypes.byref(gc), eps, _ptr(Y), _ptr(X), ld, kc, tol,
-                                     max_iter, _ptr(iters), _ptr(relres), _ptr(ws), ws.numel(),
-                                     _stream()), allow=(ERC_ERR_NOT_CONVERGED,))
-    return X, iters, relres, st
+    args = [ctypes.byref(gc), eps, _ptr(Y), _ptr(X), ld, kc, tol, max_iter, _ptr(iters),
+            _ptr(relres), _ptr(ws), ws.numel()]
+    if not timed:
+        st = _check(getattr(lib(), fn)(*args, _stream()), allow=(ERC_ERR_NOT_CONVERGED,))
+        return X, iters, relres, st
+    us = _f32(0)
+    path = _i32(0)
+    st = _check(getattr(lib(), fn)(*args, ctypes.byref(us), ctypes.byref(path), _stream()),
+                allow=(ERC_ERR_NOT_CONVERGED,))
+    return X, iters, relres, st, float(us.value), int(path.value)
+
+
+def erc_batched_cg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
+    """Returns (X, iters, relres, status); status is ERC_OK or ERC_ERR_NOT_CONVERGED."""
+    return _solve("erc_batched_cg", g, eps, Y, kc, tol, max_iter, X, ws, False)
 
 
 def erc_batched_cg_timed(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
     """erc_batched_cg plus (solve microseconds, path): 2 = cluster column-group solver, 1 = resident
     cooperative solver, 0 = multi-kernel graph loop."""
-    n, ld = Y.shape
-    dev = Y.device
-    X = torch.empty_like(Y) if X is None else X
-    iters = torch.empty(kc, dtype=torch.int32, device=dev)
-    relres = torch.empty(kc, dtype=torch.float32, device=dev)
-    if ws is None:
-        ws = _workspace(lib().erc_batched_cg_workspace_size(n, ld), dev)
-    us = _f32(0)
-    path = _i32(0)
-    gc = g.c()
-    st = _check(lib().erc_batched_cg_timed(ctypes.byref(gc), eps, _ptr(Y), _ptr(X), ld, kc, tol,
-                                           max_iter, _ptr(iters), _ptr(relres), _ptr(ws),
-                                           ws.numel(), ctypes.byref(us), ctypes.byref(path),
-                                           _stream()), allow=(ERC_ERR_NOT_CONVERGED,))
-    return X, iters, relres, st, float(us.value), int(path.value)
+    return _solve("erc_batched_cg_timed", g, eps, Y, kc, tol, max_iter, X, ws, True)
+
+
+def erc_batched_pcg(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
+    """Jacobi-preconditioned variant of erc_batched_cg (an option, not the paper's solver)."""
+    return _solve("erc_batched_pcg", g, eps, Y, kc, tol, max_iter, X, ws, False)
+
+
+def erc_batched_pcg_timed(g, eps, Y, kc, tol, max_iter=20000, X=None, ws=None):
+    """erc_batched_pcg plus (solve microseconds, path: 1 resident, 0 multi-kernel)."""
+    return _solve("erc_batched_pcg_timed", g, eps, Y, kc, tol, max_iter, X, ws, True)
 
 
 def erc_edge_resistance(g, X, kc, R_acc):
@@ -364,11 +377,13 @@ class Params:
     max_iter: int = 20000
     eta: float = 1e-8
     dup_policy: int = ERC_DUP_SUM
+    precond: int = ERC_PRECOND_NONE
 
     def c(self):
         p = ErcParamsC()
         p.seed, p.K, p.kc, p.eps, p.tol = self.seed, self.K, self.kc, self.eps, self.tol
         p.max_iter, p.eta, p.dup_policy = self.max_iter, self.eta, self.dup_policy
+        p.precond = self.precond
         return p
 
 
