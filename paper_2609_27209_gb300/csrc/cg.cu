@@ -968,8 +968,11 @@ void spmm_shape(const erc_graph* g, int ld, int* grid, int32_t* H) {
   const int gpb = T / lpr;
   *grid = one_wave_grid(spmm_kernel<MODE_STEP>(nvec, g->val != nullptr), T,
                         ((long long)g->n + gpb - 1) / gpb);
+  // rows with more neighbours than an eighth of a group's mean share go to whole blocks: on
+  // power-law graphs a group that drew a row near the mean share would otherwise hold up its
+  // block long after the others finished
   const long long groups = (long long)(*grid) * gpb;
-  long long h = 2 * g->m / (2 * groups);
+  long long h = 2 * g->m / (8 * groups);
   if (h < 32) h = 32;
   if (h > (1 << 20)) h = 1 << 20;
   *H = (int32_t)h;
