@@ -54,10 +54,44 @@ def test_binding_covers_every_declared_symbol(libpath):
 
 
 def test_library_is_built_for_sm_103a(libpath):
-    out = subprocess.run(["cuobjdump", "--list-elf", libpath], capture_output=True, text=True)
-    if out.returncode != 0:
-        pytest.skip("cuobjdump unavailable")
-    assert "sm_103a" in out.stdout
+    from paper_2609_27209_gb300 import build
+
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+    assert os.path.getmtime(libpath) >= max(
+        os.path.getmtime(os.path.join(build.CSRC, f)) for f in os.listdir(build.CSRC))
+
+
+def test_struct_layouts_match_the_header(tmp_path):
+    """sizeof and every field offset of erc_graph and erc_params, as a C compiler lays them out
+    from include/erc.h, equal the binding's ctypes structures."""
+    from paper_2609_27209_gb300 import erc
+
+    structs = {"erc_graph": erc.ErcGraphC, "erc_params": erc.ErcParamsC}
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "erc.h"', "int main(void) {"]
+    for cname, cls in structs.items():
+        lines.append(f'  printf("{cname} size %zu\\n", sizeof({cname}));')
+        for field, _ in cls._fields_:
+            lines.append(f'  printf("{cname} {field} %zu\\n", offsetof({cname}, {field}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    cc = subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o",
+                         str(exe)], capture_output=True, text=True)
+    if cc.returncode != 0 and "cuda_runtime" in cc.stderr:
+        pytest.skip("the header needs the CUDA include path")
+    assert cc.returncode == 0, cc.stderr
+    got = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    seen = 0
+    for line in got:
+        if not line:
+            continue
+        cname, field, value = line.split()
+        cls = structs[cname]
+        expect = ctypes.sizeof(cls) if field == "size" else getattr(cls, field).offset
+        assert int(value) == expect, (cname, field, value, expect)
+        seen += 1
+    assert seen == sum(len(c._fields_) + 1 for c in structs.values())
 
 
 def test_binding_fails_loudly_without_library(monkeypatch):
