@@ -142,3 +142,42 @@ def test_column_subset_matches_oracle(big):
     rel = np.abs(host(Rg).astype(np.float64) - Rr) / Rr
     assert rel.max() <= 1e-3 and np.median(rel) <= 1e-5, (rel.max(), np.median(rel))
     assert np.all(np.abs(host(iters) - itr) <= 0.1 * itr + 3)
+
+
+def test_jacobi_pcg_full_size(big):
+    """The optional Jacobi-preconditioned solve of one batch in the configuration bench.py times:
+    its true residual meets tau, it needs far fewer iterations than plain CG on these power-law
+    graphs, and its resistances equal plain CG's; on the 169k-node graph a column subset also
+    matches the oracle's preconditioned solve."""
+    n, g, prm = big["n"], big["g"], big["prm"]
+    Y = erc.erc_jl_rhs(g, prm.seed, prm.K, 0, prm.kc)
+    Xc, itc, _, stc = erc.erc_batched_cg(g, prm.eps, Y, prm.kc, prm.tol)
+    Xp, itp, rrp, stp = erc.erc_batched_pcg(g, prm.eps, Y, prm.kc, prm.tol)
+    assert stc == erc.ERC_OK and stp == erc.ERC_OK
+    AX, _ = erc.erc_laplacian_apply(g, prm.eps, Xp, prm.kc)
+    res = (Y - AX).double().norm(dim=0) / Y.double().norm(dim=0)
+    assert float(res[:prm.kc].max()) <= 2 * prm.tol, float(res.max())
+    assert 2 * int(itp.max()) <= int(itc.min()), (int(itp.max()), int(itc.min()))
+    Rc = torch.zeros(g.m, device="cuda:0")
+    Rp = torch.zeros(g.m, device="cuda:0")
+    erc.erc_edge_resistance(g, Xc, prm.kc, Rc)
+    erc.erc_edge_resistance(g, Xp, prm.kc, Rp)
+    # both solves stop at ||r|| <= tau ||y||: their resistances differ by O(tau) (the bars of
+    # the oracle parity tests, 1e-3 max and 1e-5 median at tau = 1e-6, scaled with tau)
+    rel = (Rp.double() - Rc.double()).abs() / Rc.double()
+    print(f"\n{big['name']}: PCG {int(itp.max())} vs CG {int(itc.max())} iterations; "
+          f"R max rel {float(rel.max()):.2e}, median {float(rel.median()):.2e}")
+    assert float(rel.max()) <= 1e3 * prm.tol and float(rel.median()) <= 10 * prm.tol
+    if big["name"] == "chung_lu_n169343_g2.5":
+        ref = O.build_laplacian(n, big["src"], big["dst"], big["w"])
+        kc = 8
+        Xs, its, _, st = erc.erc_batched_pcg(g, prm.eps, Y[:, :kc].contiguous(), kc, prm.tol)
+        assert st == erc.ERC_OK
+        Rg = torch.zeros(g.m, device="cuda:0")
+        erc.erc_edge_resistance(g, Xs, kc, Rg)
+        Xr, itr, _, ok = O.batched_pcg(ref, prm.eps, O.jl_rhs(ref, prm.seed, prm.K, 0, kc), prm.tol)
+        assert ok
+        Rr = O.edge_resistance(ref, Xr)
+        rel = np.abs(host(Rg).astype(np.float64) - Rr) / Rr
+        assert rel.max() <= 1e-3 and np.median(rel) <= 1e-5, (rel.max(), np.median(rel))
+        assert np.all(np.abs(host(its) - itr) <= 0.1 * itr + 3)
