@@ -51,11 +51,12 @@ def run_sharded(n, src, dst, w, params, world, rank, allreduce_sum):
     X = torch.empty_like(Y)
     status = erc.ERC_OK
 
+    solve = erc.erc_batched_pcg if params.precond == erc.ERC_PRECOND_JACOBI else erc.erc_batched_cg
+
     def shard_fn(c0, k, K_total):
         nonlocal status
         erc.erc_jl_rhs(g, params.seed, K_total, c0, k, ld=ld, out=Y)
-        _, _, _, st = erc.erc_batched_cg(g, params.eps, Y, k, params.tol, params.max_iter, X=X,
-                                         ws=ws)
+        _, _, _, st = solve(g, params.eps, Y, k, params.tol, params.max_iter, X=X, ws=ws)
         status = max(status, st)
         erc.erc_edge_resistance(g, X, k, R)
         return R
