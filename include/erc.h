@@ -291,7 +291,8 @@ erc_status erc_philox_signs(uint64_t seed, int64_t e0, int64_t e1, int32_t c0, i
  * arrays): eu, ev [m], R [m], p_node [n], kappa [m], prob_node [n], prob_edge [m], iters [K],
  * relres [K]; m_out (host).  NOT_CONVERGED is reported after all batches are done.
  * erc_run_host is the same with src, dst, w and every output in HOST memory (pinned memory
- * makes the copies asynchronous); the copies run on s inside the call.
+ * makes the copies asynchronous); the copies run on s inside the call, and every output is
+ * copied back whatever the CG status.
  * ------------------------------------------------------------------------------------------- */
 size_t erc_run_workspace_size(int32_t n, int64_t m_in, int32_t kc);
 erc_status erc_run(const erc_params* prm, int32_t n, const int32_t* src, const int32_t* dst,

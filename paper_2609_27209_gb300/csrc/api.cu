@@ -198,7 +198,8 @@ void plan_run(Arena& a, RunPlan& p, int32_t n, int64_t m_in, int32_t kc) {
 erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, const int32_t* dst,
                       const float* w, int64_t m_in, int64_t* m_out, int32_t* eu, int32_t* ev,
                       float* R, float* p_node, float* kappa, float* prob_node, float* prob_edge,
-                      int32_t* iters, float* relres, const RunPlan& p, cudaStream_t s) {
+                      int32_t* iters, float* relres, const RunPlan& p, cudaStream_t s,
+                      bool read_status = true) {
   const int32_t ld = ld_for(prm->kc);
   int64_t m = 0;
   // the build also reports whether an unweighted input kept unit weights (no merged duplicates):
@@ -224,7 +225,7 @@ erc_status run_device(const erc_params* prm, int32_t n, const int32_t* src, cons
   ERC_TRY(erc_curvature(&g, R, p_node, kappa, reinterpret_cast<erc_stream>(s)));
   ERC_TRY(erc_sampling_probs(&g, kappa, prm->eta, prob_node, prob_edge, p.aux_ws, p.aux_bytes,
                              reinterpret_cast<erc_stream>(s)));
-  return cg_status(n, ld, prm->K, prm->max_iter, p.cg_ws, s);
+  return read_status ? cg_status(n, ld, prm->K, prm->max_iter, p.cg_ws, s) : ERC_OK;
 }
 
 erc_status check_params(const erc_params* prm, int32_t n, int64_t m_in) {
@@ -334,9 +335,10 @@ extern "C" erc_status erc_run_host(const erc_params* prm, int32_t n, const int32
     ERC_CUDA(cudaMemcpyAsync(d.dst, dst, mi4, cudaMemcpyHostToDevice, s));
     if (w) ERC_CUDA(cudaMemcpyAsync(d.w, w, mi4, cudaMemcpyHostToDevice, s));
   }
-  erc_status st = run_device(prm, n, d.src, d.dst, w ? d.w : nullptr, m_in, m_out, d.eu, d.ev,
-                             d.R, d.p, d.kappa, d.pn, d.pe, d.iters, d.relres, p, s);
-  if (st != ERC_OK && st != ERC_ERR_NOT_CONVERGED) return st;
+  // the CG status is read after the output copies are enqueued: its readback is the call's one
+  // synchronisation after the build
+  ERC_TRY(run_device(prm, n, d.src, d.dst, w ? d.w : nullptr, m_in, m_out, d.eu, d.ev, d.R, d.p,
+                     d.kappa, d.pn, d.pe, d.iters, d.relres, p, s, false));
   const size_t m4 = (size_t)(*m_out) * 4, n4 = (size_t)n * 4, k4 = (size_t)prm->K * 4;
   if (m4) {
     ERC_CUDA(cudaMemcpyAsync(eu, d.eu, m4, cudaMemcpyDeviceToHost, s));
@@ -349,6 +351,5 @@ extern "C" erc_status erc_run_host(const erc_params* prm, int32_t n, const int32
   ERC_CUDA(cudaMemcpyAsync(prob_node, d.pn, n4, cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaMemcpyAsync(iters, d.iters, k4, cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaMemcpyAsync(relres, d.relres, k4, cudaMemcpyDeviceToHost, s));
-  ERC_CUDA(cudaStreamSynchronize(s));
-  return st;
+  return cg_status(n, ld_for(prm->kc), prm->K, prm->max_iter, p.cg_ws, s);
 }
