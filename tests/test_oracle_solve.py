@@ -3,11 +3,14 @@
 * Y = B^T W^{1/2} Q is compared with the dense incidence product, checked to lie in range(L)
   (1^T Y = 0 on every connected component) and checked statistically against E[Y Y^T] = L.
 * L_eps X is compared with the dense (B^T W B + eps I) X.
-* CG is compared with a direct dense solve (the paper's ERC-JL) and its true residual with tau.
+* CG is compared with a direct dense solve (the paper's ERC-JL) and its true residual with tau,
+  and its iterates (and those of the optional Jacobi PCG) step by step with scipy's cg.
 """
 import numpy as np
 import pytest
+import scipy.sparse as sp
 import scipy.sparse.csgraph as csg
+import scipy.sparse.linalg as sla
 
 from oracle import dense as D
 from oracle import erc_oracle as O
@@ -142,3 +145,26 @@ def test_pcg_needs_fewer_iterations_with_hubs():
     _, ip, rp, okp = O.batched_pcg(g, 1e-3, Y, 1e-6)
     assert okc and okp and np.all(rp <= 1.01e-6)
     assert ip.max() * 2 <= ic.max(), (ip.max(), ic.max())
+
+
+@pytest.mark.parametrize("precond", [None, "jacobi"])
+def test_iterates_match_scipy_cg(precond):
+    """After k iterations from x = 0 the oracle's CG (and Jacobi PCG) iterate equals that of
+    scipy.sparse.linalg.cg on the same L_eps and right-hand side (with the preconditioner
+    M^-1 = diag(1 / (deg + eps)) for PCG), on a power-law graph whose diagonal varies widely: the
+    alpha, beta and direction updates are pinned step by step, not only at convergence."""
+    n, src, dst, w = synth.chung_lu(400, 2.2, 2000, "unit", 3)
+    g = O.build_laplacian(n, src, dst, w)
+    A = O.adjacency(g)
+    eps = 1e-3
+    d = np.asarray(A.sum(axis=1)).ravel() + eps
+    L = sp.diags(d) - A
+    M = sla.LinearOperator((n, n), matvec=lambda v: v / d) if precond else None
+    Y = O.jl_rhs(g, 5, 4, 0, 4)
+    solve = O.batched_pcg if precond else O.batched_cg
+    for k in (1, 2, 5, 20):
+        X, iters, _, _ = solve(g, eps, Y, 1e-30, max_iter=k)
+        assert np.all(iters == k)
+        for c in range(Y.shape[1]):
+            ref, _ = sla.cg(L, Y[:, c], x0=np.zeros(n), rtol=1e-30, atol=0.0, maxiter=k, M=M)
+            assert np.linalg.norm(X[:, c] - ref) <= 1e-11 * np.linalg.norm(ref), (k, c)
