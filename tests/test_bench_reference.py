@@ -1,4 +1,4 @@
-"""bench.py's reference arm (the float64 oracle on the host cores) keeps the JSON contract: one
+"""bench.py on the CPU: the reference arm (the float64 oracle on the host cores) keeps the JSON contract: one
 line with the metric, unit, direction, config, a cpu_baseline describing the run and an e2e
 object with no host-device bytes.  Runs on the CPU, on the 2k-node workload."""
 import json
@@ -26,3 +26,33 @@ def test_reference_arm_prints_one_contract_line():
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_traffic_is_reported_only_for_the_captured_sources(tmp_path, monkeypatch):
+    """profiles/traffic.json counters are used only while the solver sources hash to the value
+    recorded with them; any other hash (a changed kernel) yields null."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    sha = bench.solver_src_sha1()
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    (prof / "traffic.json").write_text(json.dumps(
+        {"spmm": {"w1": {"dram_bytes_per_launch": 123, "solver_src_sha1": sha},
+                  "w2": {"dram_bytes_per_launch": 456, "solver_src_sha1": "0" * 40}}}))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "solver_src_sha1", lambda: sha)
+    assert bench._traffic("spmm", "w1") == 123
+    assert bench._traffic("spmm", "w2") is None
+    assert bench._traffic("spmm", "w3") is None
+    assert bench._traffic("cg_resident", "w1") is None
+
+
+def test_operator_algorithmic_bytes():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    n, m, kc = 1000, 5000, 64
+    unweighted = 4 * 2 * m + 8 * (n + 1) + 2 * 4 * n * kc
+    assert bench.spmm_algorithmic_bytes(n, m, kc, False) == unweighted
+    assert bench.spmm_algorithmic_bytes(n, m, kc, True) == unweighted + 4 * 2 * m
