@@ -1,6 +1,8 @@
-"""bench.py on the CPU: the reference arm (the float64 oracle on the host cores) keeps the JSON contract: one
-line with the metric, unit, direction, config, a cpu_baseline describing the run and an e2e
-object with no host-device bytes.  Runs on the CPU, on the 2k-node workload."""
+"""bench.py on the CPU.  The reference arm (the float64 oracle on the host cores) keeps the JSON
+contract: one line with the metric, unit, direction, config, a cpu_baseline describing the run
+and an e2e object with no host-device bytes (run on the 2k-node workload).  The ncu traffic
+counters are used only for the sources they were taken on, and the operator's algorithmic bytes
+follow their definition."""
 import json
 import os
 import subprocess
