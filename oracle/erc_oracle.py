@@ -66,7 +66,8 @@ def build_laplacian(n, src, dst, w=None, dup_policy="sum"):
     idx = np.nonzero(keep)[0]
     a = np.minimum(src[idx], dst[idx])
     b = np.maximum(src[idx], dst[idx])
-    order = np.lexsort((b, a))  # stable: equal pairs keep input order
+    # lexicographic order of (a, b) by one integer key a n + b; stable: equal pairs keep input order
+    order = np.argsort(a * n + b, kind="stable")
     a, b, wi = a[order], b[order], w_in[idx][order].astype(np.float64)
 
     if a.size:
@@ -89,7 +90,7 @@ def build_laplacian(n, src, dst, w=None, dup_policy="sum"):
     rows = np.concatenate([eu, ev])
     cols = np.concatenate([ev, eu])
     eids = np.concatenate([np.arange(m), np.arange(m)])
-    o = np.lexsort((cols, rows))
+    o = np.argsort(rows * n + cols)  # (row, col) pairs are distinct: lexicographic order
     rows, cols, eids = rows[o], cols[o], eids[o]
     row_ptr = np.zeros(n + 1, np.int64)
     np.cumsum(np.bincount(rows, minlength=n), out=row_ptr[1:])
@@ -200,11 +201,19 @@ def jl_rhs(g, seed, K, c0, kc, edge_block=1 << 16, edge_ids=None):
 # ------------------------------------------------------------------------------------------------
 
 
-def laplacian_matvec(g, eps, X, A=None):
-    """L_eps X = (D + eps I) X - A X  (Eq. 5 with L = D - A, D_uu = sum_v A_uv in float64)."""
+def laplacian_matvec(g, eps, X, A=None, d=None):
+    """L_eps X = (D + eps I) X - A X  (Eq. 5 with L = D - A, D_uu = sum_v A_uv in float64).
+
+    `d` (optional) is the diagonal D + eps I as returned by `regularised_diagonal`, passed by the
+    solvers so that it is formed once per solve rather than once per product."""
     A = adjacency(g) if A is None else A
-    d = np.asarray(A.sum(axis=1)).ravel() + eps
+    d = regularised_diagonal(A, eps) if d is None else d
     return d[:, None] * X - A @ X
+
+
+def regularised_diagonal(A, eps):
+    """The diagonal of L_eps = D - A + eps I: the float64 row sums of A plus eps (Eq. 5)."""
+    return np.asarray(A.sum(axis=1)).ravel() + eps
 
 
 def batched_cg(g, eps, Y, tol, max_iter=20000):
@@ -215,6 +224,7 @@ def batched_cg(g, eps, Y, tol, max_iter=20000):
     true relative residual ||y - L_eps x|| / ||y|| of the returned X, and `converged`.
     """
     A = adjacency(g)
+    d = regularised_diagonal(A, eps)
     Y = np.asarray(Y, dtype=np.float64)
     X = np.zeros_like(Y)
     Rv = Y.copy()
@@ -226,7 +236,7 @@ def batched_cg(g, eps, Y, tol, max_iter=20000):
     for _ in range(max_iter):
         if not active.any():
             break
-        AP = laplacian_matvec(g, eps, P, A)
+        AP = laplacian_matvec(g, eps, P, A, d)
         pAp = np.einsum("ij,ij->j", P, AP)
         alpha = np.where(active, rr / np.where(active, pAp, 1.0), 0.0)
         X += alpha * P
@@ -237,7 +247,7 @@ def batched_cg(g, eps, Y, tol, max_iter=20000):
         rr = np.where(active, rr_new, rr)
         iters += active
         active = active & (rr > (tol * tol) * yy)
-    res = Y - laplacian_matvec(g, eps, X, A)
+    res = Y - laplacian_matvec(g, eps, X, A, d)
     ny = np.sqrt(yy)
     relres = np.where(ny > 0, np.sqrt(np.einsum("ij,ij->j", res, res)) / np.where(ny > 0, ny, 1),
                       0.0)
@@ -251,7 +261,7 @@ def batched_pcg(g, eps, Y, tol, max_iter=20000):
     on the unpreconditioned recursive residual ||r|| <= tol ||y||, same outputs as batched_cg.
     """
     A = adjacency(g)
-    d = np.asarray(A.sum(axis=1)).ravel() + eps  # the diagonal of L_eps, float64
+    d = regularised_diagonal(A, eps)  # the diagonal of L_eps, float64
     Y = np.asarray(Y, dtype=np.float64)
     X = np.zeros_like(Y)
     Rv = Y.copy()
@@ -264,7 +274,7 @@ def batched_pcg(g, eps, Y, tol, max_iter=20000):
     for _ in range(max_iter):
         if not active.any():
             break
-        AP = laplacian_matvec(g, eps, P, A)
+        AP = laplacian_matvec(g, eps, P, A, d)
         pAp = np.einsum("ij,ij->j", P, AP)
         alpha = np.where(active, rz / np.where(active, pAp, 1.0), 0.0)
         X += alpha * P
@@ -277,7 +287,7 @@ def batched_pcg(g, eps, Y, tol, max_iter=20000):
         rz = np.where(active, rz_new, rz)
         iters += active
         active = active & (rr > (tol * tol) * yy)
-    res = Y - laplacian_matvec(g, eps, X, A)
+    res = Y - laplacian_matvec(g, eps, X, A, d)
     ny = np.sqrt(yy)
     relres = np.where(ny > 0, np.sqrt(np.einsum("ij,ij->j", res, res)) / np.where(ny > 0, ny, 1),
                       0.0)
