@@ -84,6 +84,19 @@ const char* erc_last_error(void);
  * counts the kernels it contains).  For instrumentation only. */
 uint64_t erc_kernel_launches(void);
 
+/* erc_set_wait_limit -- failure detection (no counterpart in the paper).  Every device-side wait
+ * of the library on work of other thread blocks of the same launch is bounded: the look-back of
+ * the single-pass scans (Laplacian build, subgraph sampler), the grid barrier of the CG vector
+ * update and the grid synchronisations of the resident CG solver.  A wait that runs out of polls
+ * records it in the call's device status and returns; the kernels after it in the same call do
+ * no further work on the unfinished result, and the call returns ERC_ERR_TIMEOUT once it reads
+ * its status (the outputs are then undefined).  `polls` sets the number of polls every such
+ * wait makes before it gives up, for all later calls of the process; 0 (the initial state)
+ * restores each wait's default, which is seconds of waiting.  Waits of work already enqueued keep
+ * the limit they were enqueued with.  The hardware cluster barriers of the cluster CG solver are
+ * not polled and take no limit. */
+void erc_set_wait_limit(uint32_t polls);
+
 /* ---------------------------------------------------------------------------------------------
  * erc_build_laplacian -- the simple undirected graph behind L = D - A = B^T W B (§3.1.1).
  *
@@ -105,6 +118,16 @@ erc_status erc_build_laplacian(int32_t n, const int32_t* src, const int32_t* dst
                                int64_t m_in, int32_t dup_policy, int64_t* row_ptr, int32_t* col,
                                float* val, float* deg, int32_t* csr_eid, int32_t* eu, int32_t* ev,
                                float* ew, int64_t* m_out, void* ws, size_t ws_bytes, erc_stream s);
+/* erc_build_laplacian_ex -- erc_build_laplacian, plus *unit_weights (host) = 1 when w is NULL and
+ * no merged duplicate pair received a weight other than 1, else 0.  When it is 1 every weight of
+ * the graph is 1: an erc_graph may then carry val = ew = NULL, and the kernels read neighbour
+ * indices only.  The flag comes back with m_out in the same synchronisation. */
+erc_status erc_build_laplacian_ex(int32_t n, const int32_t* src, const int32_t* dst,
+                                  const float* w, int64_t m_in, int32_t dup_policy,
+                                  int64_t* row_ptr, int32_t* col, float* val, float* deg,
+                                  int32_t* csr_eid, int32_t* eu, int32_t* ev, float* ew,
+                                  int64_t* m_out, int32_t* unit_weights, void* ws,
+                                  size_t ws_bytes, erc_stream s);
 
 /* ---------------------------------------------------------------------------------------------
  * erc_jl_rhs -- Y[:, 0:kc] = (B^T W^{1/2} Q)[:, c0:c0+kc]  (§3.1.2; Algorithm 1 "form Y").
@@ -209,7 +232,8 @@ erc_status erc_sampling_probs(const erc_graph* g, const float* kappa, float eta,
  * the library and held until the process exits.  The call allocates nothing.
  * Limits: g->n <= ERC_SAMPLING_PROBS_NOALLOC_MAX_NODES, else ERC_ERR_CAPACITY (nothing is run).
  * The first call on each device looks up the array's device address (cudaGetSymbolAddress) with
- * that device current; make that first call before any stream capture.  All calls share the one
+ * that device current, and so does the first call after the device's context was destroyed and
+ * created again (cudaDeviceReset): make those calls before any stream capture.  All calls share the one
  * array and it keeps the last call's contents (a call never relies on them): calls that may
  * overlap on the GPU -- concurrent streams, or several host threads -- race with each other and
  * must be serialised by the caller.

@@ -16,6 +16,12 @@ thread_local char g_err[512] = "";
 thread_local bool g_capturing = false;
 thread_local long long g_captured = 0;  // kernels recorded into the graph being captured
 std::atomic<unsigned long long> g_launches{0};
+std::atomic<unsigned> g_wait_limit{0};  // 0: every bounded wait keeps its own default
+}
+
+unsigned wait_limit(unsigned dflt) {
+  const unsigned v = g_wait_limit.load(std::memory_order_relaxed);
+  return v ? v : dflt;
 }
 
 void count_launches(long long k) {
@@ -247,6 +253,9 @@ using namespace erc;
 extern "C" const char* erc_version(void) { return "erc-gb300 0.1 (sm_103a)"; }
 extern "C" const char* erc_last_error(void) { return g_err; }
 extern "C" uint64_t erc_kernel_launches(void) { return g_launches.load(); }
+extern "C" void erc_set_wait_limit(uint32_t polls) {
+  g_wait_limit.store(polls, std::memory_order_relaxed);
+}
 
 extern "C" size_t erc_run_workspace_size(int32_t n, int64_t m_in, int32_t kc) {
   if (n < 1 || m_in < 0 || kc < 1) return 0;

@@ -20,7 +20,8 @@ struct BuildPlan {
   int32_t* row_of;
   float* wmerged;
   int64_t* counters;  // [0] nnz  [1] m
-  unsigned* err;      // bit 0: node id out of range, bit 1: bad weight
+  unsigned* err;      // [0] bit 0: node id out of range, bit 1: bad weight; [1] a merged
+                      // weight differs from 1; [2] the abort word (a scan's wait gave up)
   void *sort_tmp, *scan_tmp;
 };
 
@@ -72,7 +73,8 @@ __global__ void k_emit(const int32_t* __restrict__ src, const int32_t* __restric
 }
 
 __global__ void k_heads(const uint64_t* __restrict__ keys, int64_t E, uint64_t sent,
-                        uint8_t* __restrict__ head) {
+                        uint8_t* __restrict__ head, const unsigned* abort) {
+  if (aborted(abort)) return;  // the sort did not finish: nothing after it runs
   for (int64_t i = gtid(); i < E; i += gstride()) {
     uint64_t k = keys[i];
     head[i] = (k != sent) && (i == 0 || keys[i - 1] != k);
@@ -86,7 +88,8 @@ __global__ void k_emit_csr(const uint64_t* __restrict__ keys, const uint32_t* __
                            const float* __restrict__ w, int64_t E, int B, int dup_first,
                            int32_t* __restrict__ col, float* __restrict__ wmerged,
                            int32_t* __restrict__ row_of, uint8_t* __restrict__ upper,
-                           unsigned* __restrict__ nonunit) {
+                           unsigned* __restrict__ nonunit, const unsigned* abort) {
+  if (aborted(abort)) return;
   const uint64_t mask = (1ull << B) - 1ull;
   bool other = false;
   for (int64_t i = gtid(); i < E; i += gstride()) {
@@ -111,7 +114,8 @@ __global__ void k_emit_csr(const uint64_t* __restrict__ keys, const uint32_t* __
 }
 
 __global__ void k_row_ptr(const int32_t* __restrict__ row_of, const int64_t* __restrict__ counters,
-                          int32_t n, int64_t* __restrict__ row_ptr) {
+                          int32_t n, int64_t* __restrict__ row_ptr, const unsigned* abort) {
+  if (aborted(abort)) return;
   const int64_t nnz = counters[0];
   for (int64_t s = gtid(); s < nnz; s += gstride()) {
     int32_t r = row_of[s];
@@ -124,7 +128,8 @@ __global__ void k_row_ptr(const int32_t* __restrict__ row_of, const int64_t* __r
 
 __global__ void k_degree(const int64_t* __restrict__ row_ptr, const float* __restrict__ wmerged,
                          int32_t n, float* __restrict__ deg, float* __restrict__ val,
-                         const int64_t* __restrict__ counters) {
+                         const int64_t* __restrict__ counters, const unsigned* abort) {
+  if (aborted(abort)) return;
   for (int64_t r = gtid(); r < n; r += gstride()) {
     double acc = 0.0;  // sequential float64 sum in column order
     for (int64_t j = row_ptr[r]; j < row_ptr[r + 1]; ++j) {
@@ -141,7 +146,8 @@ __global__ void k_emit_edges(const uint8_t* __restrict__ upper, const int64_t* _
                              const float* __restrict__ wmerged,
                              const int64_t* __restrict__ counters, int32_t* __restrict__ eu,
                              int32_t* __restrict__ ev, float* __restrict__ ew,
-                             int32_t* __restrict__ csr_eid) {
+                             int32_t* __restrict__ csr_eid, const unsigned* abort) {
+  if (aborted(abort)) return;
   const int64_t nnz = counters[0];
   for (int64_t s = gtid(); s < nnz; s += gstride()) {
     if (!upper[s]) continue;
@@ -155,7 +161,9 @@ __global__ void k_emit_edges(const uint8_t* __restrict__ upper, const int64_t* _
 
 __global__ void k_lower_eid(const uint8_t* __restrict__ upper, const int32_t* __restrict__ row_of,
                             const int32_t* __restrict__ col, const int64_t* __restrict__ row_ptr,
-                            const int64_t* __restrict__ counters, int32_t* __restrict__ csr_eid) {
+                            const int64_t* __restrict__ counters, int32_t* __restrict__ csr_eid,
+                            const unsigned* abort) {
+  if (aborted(abort)) return;
   const int64_t nnz = counters[0];
   for (int64_t s = gtid(); s < nnz; s += gstride()) {
     if (upper[s]) continue;
@@ -215,6 +223,7 @@ erc_status erc::build_laplacian_impl(int32_t n, const int32_t* src, const int32_
   const int64_t E = 2 * m_in;
   const int B = bit_length((uint32_t)n);  // 2^B > n - 1: every id fits, and the sentinel sorts last
   const uint64_t sent = (2 * B >= 64) ? ~0ull : ((1ull << (2 * B)) - 1ull);
+  unsigned* abort = p.err + 2;
   auto enqueue = [&](cudaStream_t cs) -> erc_status {
     ERC_CUDA(cudaMemsetAsync(p.counters, 0, 4 * sizeof(int64_t), cs));
     ERC_CUDA(cudaMemsetAsync(p.err, 0, 4 * sizeof(unsigned), cs));
@@ -224,32 +233,36 @@ erc_status erc::build_laplacian_impl(int32_t n, const int32_t* src, const int32_
                                                 p.err);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
-      ERC_TRY(radix_sort_pairs(p.keys, p.vals, p.keys_alt, p.vals_alt, E, 2 * B, p.sort_tmp, cs));
-      k_heads<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, E, sent, p.head);
+      ERC_TRY(radix_sort_pairs(p.keys, p.vals, p.keys_alt, p.vals_alt, E, 2 * B, p.sort_tmp, cs,
+                               abort));
+      k_heads<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, E, sent, p.head, abort);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
-      ERC_TRY(exclusive_scan_i64(nullptr, p.head, p.slot, E, &p.counters[0], p.scan_tmp, cs));
+      ERC_TRY(exclusive_scan_i64(nullptr, p.head, p.slot, E, &p.counters[0], p.scan_tmp, cs,
+                                 abort));
       ERC_CUDA(cudaMemsetAsync(p.upper, 0, (size_t)E, cs));  // slots past nnz must not count
       k_emit_csr<<<grid_for(E, BT), BT, 0, cs>>>(p.keys, p.vals, p.head, p.slot, w, E, B,
                                                 dup_policy == ERC_DUP_FIRST, col, p.wmerged,
-                                                p.row_of, p.upper, w ? nullptr : p.err + 1);
+                                                p.row_of, p.upper, w ? nullptr : p.err + 1,
+                                                abort);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
-      k_row_ptr<<<grid_for(E, BT), BT, 0, cs>>>(p.row_of, p.counters, n, row_ptr);
+      k_row_ptr<<<grid_for(E, BT), BT, 0, cs>>>(p.row_of, p.counters, n, row_ptr, abort);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
     }
-    k_degree<<<grid_for(n, BT), BT, 0, cs>>>(row_ptr, p.wmerged, n, deg, val, p.counters);
+    k_degree<<<grid_for(n, BT), BT, 0, cs>>>(row_ptr, p.wmerged, n, deg, val, p.counters, abort);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
     if (m_in > 0) {
-      ERC_TRY(exclusive_scan_i64(nullptr, p.upper, p.eidx, E, &p.counters[1], p.scan_tmp, cs));
+      ERC_TRY(exclusive_scan_i64(nullptr, p.upper, p.eidx, E, &p.counters[1], p.scan_tmp, cs,
+                                 abort));
       k_emit_edges<<<grid_for(E, BT), BT, 0, cs>>>(p.upper, p.eidx, p.row_of, col, p.wmerged,
-                                                  p.counters, eu, ev, ew, csr_eid);
+                                                  p.counters, eu, ev, ew, csr_eid, abort);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
       k_lower_eid<<<grid_for(E, BT), BT, 0, cs>>>(p.upper, p.row_of, col, row_ptr, p.counters,
-                                                 csr_eid);
+                                                 csr_eid, abort);
       count_launches(1);
       ERC_CUDA(cudaGetLastError());
     }
@@ -258,12 +271,16 @@ erc_status erc::build_laplacian_impl(int32_t n, const int32_t* src, const int32_
   GraphKey key;
   key.add((uint64_t)n).add((uint64_t)m_in).add((uint64_t)dup_policy).add(src).add(dst).add(w);
   key.add(row_ptr).add(col).add(val).add(deg).add(csr_eid).add(eu).add(ev).add(ew).add(a.base);
+  key.add((uint64_t)wait_limit(0));
   ERC_TRY(graph_launch(key, enqueue, s));
   int64_t h_counters[2] = {0, 0};
-  unsigned h_err[2] = {0, 0};
+  unsigned h_err[3] = {0, 0, 0};
   ERC_CUDA(cudaMemcpyAsync(h_counters, p.counters, 2 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
-  ERC_CUDA(cudaMemcpyAsync(h_err, p.err, 2 * sizeof(unsigned), cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(h_err, p.err, 3 * sizeof(unsigned), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
+  if (h_err[2])
+    return set_error(ERC_ERR_TIMEOUT, "a bounded wait in the Laplacian build's scans ran out; "
+                                      "the outputs are undefined");
   if (h_err[0] & 1u) return set_error(ERC_ERR_INVALID_ARG, "node id outside [0, %d)", n);
   if (h_err[0] & 2u) return set_error(ERC_ERR_INVALID_ARG, "edge weight not finite and positive");
   if (h_counters[0] != 2 * h_counters[1])
@@ -283,4 +300,20 @@ extern "C" erc_status erc_build_laplacian(int32_t n, const int32_t* src, const i
   clear_error();
   return build_laplacian_impl(n, src, dst, w, m_in, dup_policy, row_ptr, col, val, deg, csr_eid,
                               eu, ev, ew, m_out, ws, ws_bytes, as_stream(stream), nullptr);
+}
+
+extern "C" erc_status erc_build_laplacian_ex(int32_t n, const int32_t* src, const int32_t* dst,
+                                             const float* w, int64_t m_in, int32_t dup_policy,
+                                             int64_t* row_ptr, int32_t* col, float* val,
+                                             float* deg, int32_t* csr_eid, int32_t* eu,
+                                             int32_t* ev, float* ew, int64_t* m_out,
+                                             int32_t* unit_weights, void* ws, size_t ws_bytes,
+                                             erc_stream stream) {
+  clear_error();
+  ERC_REQUIRE(unit_weights, "unit_weights is required");
+  int nonunit = 1;
+  ERC_TRY(build_laplacian_impl(n, src, dst, w, m_in, dup_policy, row_ptr, col, val, deg, csr_eid,
+                               eu, ev, ew, m_out, ws, ws_bytes, as_stream(stream), &nonunit));
+  *unit_weights = nonunit ? 0 : 1;
+  return ERC_OK;
 }

@@ -6,9 +6,10 @@
 //                      light row (float4 along the columns); rows heavier than H are taken by a
 //                      whole block, its groups splitting the row and combining in a fixed order.
 //                      Per-column p.Ap partials; the last block to finish forms alpha = rr / pAp.
-//   k_update_fused     x += alpha p, r -= alpha Ap and r.r; the last block forms beta, counts the
-//                      iteration and retires converged columns, then releases a grid barrier;
-//                      every block then applies p = r + beta p to its rows.  Launched
+//   k_update_fused     r -= alpha Ap and r.r; the last block forms beta, counts the iteration
+//                      and retires converged columns, then releases a grid barrier; every block
+//                      then applies x += alpha p and p = r + beta p to its rows (x's update reads
+//                      the p it needs there: 8 vector passes instead of 9).  Launched
 //                      cooperatively (all blocks resident), the barrier wait is bounded.
 // Reductions are deterministic: fixed groupings and orders, float-pair accumulation.  S
 // iterations are captured once into a CUDA graph and relaunched; kernels return at once when no
@@ -24,19 +25,15 @@ namespace erc {
 namespace {
 
 struct HeavyRows {
-  uint8_t* flag;    // [n]
-  int64_t* pos;     // [n]
   int32_t* list;    // [n] rows with more than H neighbours, ascending
   int64_t* count;   // [1]
-  void* scan_tmp;
+  int* bcount;      // [MAX_GRID] heavy rows in each listing block's range of rows
 };
 
 void plan_heavy(Arena& a, HeavyRows& h, int32_t n) {
-  h.flag = a.take<uint8_t>(n);
-  h.pos = a.take<int64_t>(n);
   h.list = a.take<int32_t>(n);
   h.count = a.take<int64_t>(1);
-  h.scan_tmp = a.take<char>(scan_temp_bytes(n));
+  h.bcount = a.take<int>(MAX_GRID);
 }
 
 struct CgWork {
@@ -118,7 +115,9 @@ __device__ __forceinline__ void load_row(const SpmmArgs& a, int64_t u, int gl, i
 
 template <int LPR, int VPL, bool WEIGHTED, int MODE>
 __global__ void __launch_bounds__(T, VPL <= 2 ? 3 : VPL == 4 ? 2 : 1) k_spmm(SpmmArgs a) {
-  if (MODE == MODE_STEP && *(volatile int*)a.flags == 0) return;
+  // nothing left to do: no active column, or a bounded wait of the solve has given up
+  if (MODE == MODE_STEP && (*(volatile int*)a.flags == 0 || *(volatile int*)(a.flags + 3) != 0))
+    return;
   __shared__ __align__(16) float smem[SMEM_FLOATS];
   constexpr int GPB = T / LPR;  // groups per block
   const int gl = threadIdx.x & (LPR - 1);
@@ -296,11 +295,15 @@ __global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
   if (threadIdx.x == 0) a.flags[0] = any;
 }
 
-// x += alpha p, r -= alpha Ap, r.r  |grid barrier: beta, convergence|  p = r + beta p
+// r -= alpha Ap, r.r  |grid barrier: beta, convergence|  x += alpha p, p = r + beta p
+// The x update uses this iteration's alpha and the p it was formed with, exactly as it would
+// before the barrier, so the iterates do not change; it is applied after the barrier because
+// that pass reads p anyway (x, p, r read; x, p written: with r, Ap read and r written before
+// the barrier, 8 passes over the n x ld block).
 // With the Jacobi preconditioner (a.deg set) the first part also sums r.z, z = r / (deg + eps),
 // beta is the ratio of successive r.z, and p = z + beta p; the stop test stays on r.r.
 __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
-  if (*(volatile int*)a.flags == 0) return;
+  if (*(volatile int*)a.flags == 0 || *(volatile int*)(a.flags + 3) != 0) return;
   __shared__ float2 red[T * 4];
   __shared__ float2 sbuf[2 * MAX_LD];
   const bool pc = a.deg != nullptr;
@@ -318,19 +321,12 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   if (al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f) {
     for (int64_t row = row0; row < a.n; row += rstep) {
       const size_t i = (size_t)row * a.ld + 4 * q;
-      float4 x = *reinterpret_cast<const float4*>(a.X + i);
       float4 r = *reinterpret_cast<const float4*>(a.R + i);
-      const float4 p = *reinterpret_cast<const float4*>(a.P + i);
       const float4 ap = *reinterpret_cast<const float4*>(a.AP + i);
-      x.x = fmaf(al.x, p.x, x.x);
-      x.y = fmaf(al.y, p.y, x.y);
-      x.z = fmaf(al.z, p.z, x.z);
-      x.w = fmaf(al.w, p.w, x.w);
       r.x = fmaf(-al.x, ap.x, r.x);
       r.y = fmaf(-al.y, ap.y, r.y);
       r.z = fmaf(-al.z, ap.z, r.z);
       r.w = fmaf(-al.w, ap.w, r.w);
-      *reinterpret_cast<float4*>(a.X + i) = x;
       *reinterpret_cast<float4*>(a.R + i) = r;
       d[0] = df_fma(d[0], r.x, r.x);
       d[1] = df_fma(d[1], r.y, r.y);
@@ -382,7 +378,7 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   } else if (threadIdx.x == 0) {
     unsigned spins = 0;
     while (ld_acquire(a.gen) == s_gen) {
-      if (++spins > SPIN_LIMIT) {  // bounded: flag the timeout and fall through
+      if (++spins > a.spin_limit) {  // bounded: flag the timeout and fall through
         atomicOr(&a.flags[3], 1);
         break;
       }
@@ -390,14 +386,27 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
     }
   }
   __syncthreads();
+  // columns with alpha != 0 were active in this iteration: x += alpha p; those still active
+  // after it: p = r + beta p (a column that converged now still takes its last x update)
   const int4 act = __ldcg(reinterpret_cast<const int4*>(a.active + 4 * q));
-  if (!(act.x | act.y | act.z | act.w)) return;
   const float4 be = __ldcg(reinterpret_cast<const float4*>(a.beta + 4 * q));
+  const bool any_p = act.x | act.y | act.z | act.w;
+  const bool any_x = al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f;
+  if (!any_x && !any_p) return;
   for (int64_t row = row0; row < a.n; row += rstep) {
     const size_t i = (size_t)row * a.ld + 4 * q;
+    float4 p = *reinterpret_cast<const float4*>(a.P + i);
+    if (any_x) {
+      float4 x = *reinterpret_cast<const float4*>(a.X + i);
+      x.x = fmaf(al.x, p.x, x.x);
+      x.y = fmaf(al.y, p.y, x.y);
+      x.z = fmaf(al.z, p.z, x.z);
+      x.w = fmaf(al.w, p.w, x.w);
+      *reinterpret_cast<float4*>(a.X + i) = x;
+    }
+    if (!any_p) continue;
     float4 r = *reinterpret_cast<const float4*>(a.R + i);
     if (pc) r = f4_scale(r, jacobi_inv(a.deg, row, a.eps));  // z
-    float4 p = *reinterpret_cast<const float4*>(a.P + i);
     if (act.x) p.x = fmaf(be.x, p.x, r.x);
     if (act.y) p.y = fmaf(be.y, p.y, r.y);
     if (act.z) p.z = fmaf(be.z, p.z, r.z);
@@ -932,17 +941,58 @@ __global__ void __launch_bounds__(CT, 1) k_cg_cluster(ClusterArgs a) {
 }
 
 // ---------------------------------------------------------------------------- heavy rows
-__global__ void k_mark_heavy(const int64_t* __restrict__ row_ptr, int32_t n, int32_t H,
-                             uint8_t* __restrict__ flag) {
-  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n;
-       u += (int64_t)gridDim.x * blockDim.x)
-    flag[u] = (row_ptr[u + 1] - row_ptr[u]) > H;
+// The rows with more than H neighbours, ascending, in two launches and without any wait between
+// blocks: block b first counts the heavy rows of its contiguous range [b per, (b + 1) per), then
+// writes them, in order, after the counts of the blocks before it.  Integer counts: the list does
+// not depend on timing.
+constexpr int HLT = 256;
+
+__global__ void __launch_bounds__(HLT) k_count_heavy(const int64_t* __restrict__ row_ptr,
+                                                     int32_t n, int32_t H, int64_t per,
+                                                     int* __restrict__ bcount) {
+  __shared__ int s_cnt;
+  if (threadIdx.x == 0) s_cnt = 0;
+  __syncthreads();
+  const int64_t u0 = (int64_t)blockIdx.x * per, u1 = min((int64_t)n, u0 + per);
+  int c = 0;
+  for (int64_t u = u0 + threadIdx.x; u < u1; u += HLT) c += (row_ptr[u + 1] - row_ptr[u]) > H;
+  if (c) atomicAdd(&s_cnt, c);
+  __syncthreads();
+  if (threadIdx.x == 0) bcount[blockIdx.x] = s_cnt;
 }
-__global__ void k_list_heavy(const uint8_t* __restrict__ flag, const int64_t* __restrict__ pos,
-                             int32_t n, int32_t* __restrict__ list) {
-  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n;
-       u += (int64_t)gridDim.x * blockDim.x)
-    if (flag[u]) list[pos[u]] = (int32_t)u;
+
+__global__ void __launch_bounds__(HLT) k_list_heavy(const int64_t* __restrict__ row_ptr,
+                                                    int32_t n, int32_t H, int64_t per,
+                                                    const int* __restrict__ bcount,
+                                                    int32_t* __restrict__ list,
+                                                    int64_t* __restrict__ count) {
+  __shared__ unsigned long long s_off;
+  __shared__ int s_wcnt[HLT / 32];
+  if (threadIdx.x == 0) s_off = 0;
+  __syncthreads();
+  unsigned long long o = 0;
+  for (int b = threadIdx.x; b < (int)blockIdx.x; b += HLT) o += (unsigned)bcount[b];
+  if (o) atomicAdd(&s_off, o);
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t u0 = (int64_t)blockIdx.x * per, u1 = min((int64_t)n, u0 + per);
+  int64_t off = (int64_t)s_off;
+  for (int64_t base = u0; base < u1; base += HLT) {
+    const int64_t u = base + threadIdx.x;
+    const bool heavy = u < u1 && row_ptr[u + 1] - row_ptr[u] > H;
+    const unsigned bal = __ballot_sync(0xffffffffu, heavy);
+    if (lane == 0) s_wcnt[warp] = __popc(bal);
+    __syncthreads();
+    int64_t mine = off, tot = 0;
+    for (int w = 0; w < HLT / 32; ++w) {
+      if (w < warp) mine += s_wcnt[w];
+      tot += s_wcnt[w];
+    }
+    if (heavy) list[mine + __popc(bal & ((1u << lane) - 1u))] = (int32_t)u;
+    off += tot;
+    __syncthreads();
+  }
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) *count = off;
 }
 
 // ---------------------------------------------------------------------------- launch helpers
@@ -979,12 +1029,12 @@ void spmm_shape(const erc_graph* g, int ld, int* grid, int32_t* H) {
 }
 
 erc_status build_heavy(const erc_graph* g, int32_t H, const HeavyRows& hv, cudaStream_t s) {
-  const int grid = grid_for(g->n, 256);
-  k_mark_heavy<<<grid, 256, 0, s>>>(g->row_ptr, g->n, H, hv.flag);
+  const int grid = grid_for(g->n, 8 * HLT);  // at most 8 SMs' worth of blocks per SM, <= MAX_GRID
+  const int64_t per = ((int64_t)g->n + grid - 1) / grid;
+  k_count_heavy<<<grid, HLT, 0, s>>>(g->row_ptr, g->n, H, per, hv.bcount);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
-  ERC_TRY(exclusive_scan_i64(nullptr, hv.flag, hv.pos, g->n, hv.count, hv.scan_tmp, s));
-  k_list_heavy<<<grid, 256, 0, s>>>(hv.flag, hv.pos, g->n, hv.list);
+  k_list_heavy<<<grid, HLT, 0, s>>>(g->row_ptr, g->n, H, per, hv.bcount, hv.list, hv.count);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
@@ -1249,11 +1299,11 @@ erc_status launch_iteration(const SpmmArgs& sa, int sgrid, const VecArgs& va, in
 // ---------------------------------------------------------------------------- graph cache
 struct GraphKey {
   const void* ptr[15];
-  long long num[10];
+  long long num[11];
   bool operator==(const GraphKey& o) const {
     for (int i = 0; i < 15; ++i)
       if (ptr[i] != o.ptr[i]) return false;
-    for (int i = 0; i < 10; ++i)
+    for (int i = 0; i < 11; ++i)
       if (num[i] != o.num[i]) return false;
     return true;
   }
@@ -1289,9 +1339,9 @@ erc_status iteration_graph(const SpmmArgs& sa, int sgrid, const VecArgs& va, int
   long long tol_bits = 0;
   memcpy(&eps_bits, &sa.eps, sizeof eps_bits);
   memcpy(&tol_bits, &va.tol2, sizeof tol_bits);
-  long long nums[10] = {sa.n, sa.ld, sa.kc, eps_bits, tol_bits, va.max_iter, S, dev, sgrid,
-                        (long long)ugrid << 32 | (unsigned)sa.H};
-  for (int i = 0; i < 10; ++i) k.num[i] = nums[i];
+  long long nums[11] = {sa.n, sa.ld, sa.kc, eps_bits, tol_bits, va.max_iter, S, dev, sgrid,
+                        (long long)ugrid << 32 | (unsigned)sa.H, (long long)va.spin_limit};
+  for (int i = 0; i < 11; ++i) k.num[i] = nums[i];
   std::lock_guard<std::mutex> lock(g_mu);
   ++g_clock;
   int victim = 0;
@@ -1406,6 +1456,7 @@ erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float*
   va.cr = w.cr;
   va.deg = precond ? g->deg : nullptr;
   va.eps = eps;
+  va.spin_limit = wait_limit(SPIN_LIMIT);
 
   SpmmArgs sa{};
   sa.row_ptr = g->row_ptr;
@@ -1482,20 +1533,21 @@ erc_status erc::cg_enqueue(const erc_graph* g, float eps, const float* Y, float*
   } else if (resident) {
     // the whole solve in one cooperative launch, no host round trips
     ResArgs ra{sa, va, rb};
+    ra.v.spin_limit = wait_limit(RES_SPIN_LIMIT);
     ERC_TRY(launch_resident(kres, ra, smem, s));
   } else {
     const int S = iterations_per_poll(g, ld);
     cudaGraphExec_t exec = nullptr;
     ERC_TRY(iteration_graph(sa, sgrid, va, ugrid, S, &exec));
     int done = 0;
-    int h_any = 1;
+    int h_flags[4] = {1, 0, 0, 0};
     while (done < max_iter) {
       ERC_CUDA(cudaGraphLaunch(exec, s));
       count_launches(2LL * S);  // the graph holds S iterations of two kernels
       done += S;
-      ERC_CUDA(cudaMemcpyAsync(&h_any, w.flags, sizeof(int), cudaMemcpyDeviceToHost, s));
+      ERC_CUDA(cudaMemcpyAsync(h_flags, w.flags, 4 * sizeof(int), cudaMemcpyDeviceToHost, s));
       ERC_CUDA(cudaStreamSynchronize(s));
-      if (!h_any) break;
+      if (!h_flags[0] || h_flags[3]) break;  // every column stopped, or a wait gave up
     }
   }
   if (ev1) ERC_CUDA(cudaEventRecord(ev1, s));

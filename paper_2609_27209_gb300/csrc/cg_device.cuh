@@ -12,7 +12,11 @@ namespace {
 constexpr int T = 256;
 constexpr int WARPS = T / 32;
 constexpr int SMEM_FLOATS = 8192;  // 32 KB: heavy-row combine buffer, or the reduction buffers
+// default poll limits of the bounded waits: the vector update's grid barrier (which sleeps 64 ns
+// between polls) and the resident solver's synchronisations (one L2 round trip per poll); either
+// is seconds, far beyond any legitimate wait
 constexpr unsigned SPIN_LIMIT = 1u << 24;
+constexpr unsigned RES_SPIN_LIMIT = 1u << 22;
 enum { MODE_STEP = 0, MODE_APPLY = 1, MODE_RESID = 2 };
 
 struct SpmmArgs {
@@ -190,6 +194,7 @@ struct VecArgs {
   // null for plain CG
   const float* deg;
   float eps;
+  unsigned spin_limit;  // polls of a bounded wait before it gives up (sets flags[3])
 };
 
 // 1 / (deg_u + eps), the inverse diagonal of L_eps at row u
@@ -243,12 +248,13 @@ __device__ __forceinline__ void res_arrive(unsigned* arr) {
   __syncthreads();
   if (threadIdx.x == 0) red_release_add(arr, 1u);
 }
-// bounded wait until `target` arrivals (sets flags[3] on timeout)
-__device__ __forceinline__ void res_wait(const unsigned* arr, unsigned target, int* flags) {
+// bounded wait until `target` arrivals: after `limit` polls it sets flags[3] and returns
+__device__ __forceinline__ void res_wait(const unsigned* arr, unsigned target, int* flags,
+                                         unsigned limit) {
   if (threadIdx.x == 0) {
     unsigned spins = 0;
-    while ((int)(ld_acquire(arr) - target) < 0) {  // one L2 round trip per poll: ~2^22 is seconds
-      if (++spins > (1u << 22)) {
+    while ((int)(ld_acquire(arr) - target) < 0) {  // one L2 round trip per poll
+      if (++spins > limit) {
         atomicOr(&flags[3], 1);
         break;
       }
@@ -358,10 +364,10 @@ __device__ __forceinline__ void block_apply(const SpmmArgs& a, const float* src_
 // part), count in, wait for every block, then sum all blocks' rows in a fixed order into sbuf
 __device__ __forceinline__ void res_reduce(float2* part, int ld, const float2* bpart,
                                            float2* sbuf, float2* scratch, unsigned* arrivals,
-                                           unsigned& nsync, int* flags) {
+                                           unsigned& nsync, int* flags, unsigned limit) {
   for (int c = threadIdx.x; c < ld; c += PT) part[(size_t)blockIdx.x * ld + c] = bpart[c];
   res_arrive(arrivals);
-  res_wait(arrivals, ++nsync * gridDim.x, flags);
+  res_wait(arrivals, ++nsync * gridDim.x, flags, limit);
   colsum_rows(part, gridDim.x, ld, sbuf, scratch);
 }
 
@@ -480,12 +486,13 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dz, sbuf, scratch, ld);
     for (int c = threadIdx.x; c < ld; c += PT) part_yz[(size_t)blockIdx.x * ld + c] = sbuf[c];
     res_arrive(arrivals);
-    res_wait(arrivals, ++nsync * G, va.flags);
+    res_wait(arrivals, ++nsync * G, va.flags, va.spin_limit);
     colsum_rows(part_yz, G, ld, sbuf, scratch);
     for (int c = threadIdx.x; c < ld; c += PT) s_rr[c] = sbuf[c];
     colsum_rows(part_init, G, ld, sbuf, scratch);
   } else {
-    res_reduce(part_init, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);  // also publishes p
+    res_reduce(part_init, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags,
+               va.spin_limit);  // also publishes p
   }
   int any = 0;
   for (int c = threadIdx.x; c < ld; c += PT) {
@@ -515,7 +522,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
   while (any) {
     if (*(volatile int*)&va.flags[3] != 0) break;
     // ---------------- A: Ap = L_eps p on own rows, p.Ap
-    if (nsync > 1) res_wait(arrivals, nsync * G, va.flags);  // every block's p is written
+    if (nsync > 1) res_wait(arrivals, nsync * G, va.flags, va.spin_limit);  // every p written
     // this lane's float4 slots with an active column: converged columns are neither gathered
     // nor updated (their alpha is 0)
     unsigned on = 0;
@@ -541,7 +548,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
           dot[v][3] = df_fma(dot[v][3], pu.w, o.w);
         });
     block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-    res_reduce(part_pap, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);
+    res_reduce(part_pap, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags, va.spin_limit);
     for (int c = threadIdx.x; c < ld; c += PT) {
       const float2 v = sbuf[c];
       float al = 0.f;
@@ -627,7 +634,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         part_rz[(size_t)blockIdx.x * ld + c] = __fadd_rn(sbuf[c].x, sbuf[c].y);
     }
     res_arrive(arrivals);
-    res_wait(arrivals, ++nsync * G, va.flags);
+    res_wait(arrivals, ++nsync * G, va.flags, va.spin_limit);
     if constexpr (PC) {
       colsum_rows_f(part_rz, G, ld, sbuf, scratch);
       for (int c = threadIdx.x; c < ld; c += PT) s_rz[c] = sbuf[c];
@@ -729,7 +736,7 @@ __global__ void __launch_bounds__(PT, 1) k_cg_resident(ResArgs ra) {
         dot[v][3] = df_fma(dot[v][3], rw, rw);
       });
   block_partials_groups<LPR, VPL, PWARPS, PCH>(dot, sbuf, scratch, ld);
-  res_reduce(part_res, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags);
+  res_reduce(part_res, ld, sbuf, sbuf, scratch, arrivals, nsync, va.flags, va.spin_limit);
   if (blockIdx.x == 0)
     for (int c = threadIdx.x; c < a.kc; c += PT) {
       const float q = s_yy[c].x > 0.f ? df_div(sbuf[c], s_yy[c]) : 0.f;

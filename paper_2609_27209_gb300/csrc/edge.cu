@@ -387,23 +387,57 @@ static __device__ __align__(256) unsigned char g_probs_noalloc_scratch[ERC_SAMPL
 
 namespace erc {
 namespace {
-// The array's device address, looked up once per device with that device current.  In host code
-// the symbol names a host-side stand-in, never the device memory, so kernels only ever receive
-// this looked-up address.
+// The identity of the calling thread's current CUDA context (cuCtxGetId, reached through the
+// runtime's driver entry points so that the library does not link the driver library): 0 when
+// it cannot be read.  Context ids are never reused within a process.
+unsigned long long current_context_id() {
+  using GetCurrent = int (*)(void**);
+  using GetId = int (*)(void*, unsigned long long*);
+  static GetCurrent get_current = nullptr;
+  static GetId get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrent>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetId>(f);
+    cudaGetLastError();
+  });
+  void* ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != 0 || !ctx || get_id(ctx, &id) != 0) return 0;
+  return id;
+}
+
+// The array's device address, looked up with cudaGetSymbolAddress the first time a device is used
+// in a context and cached under (device, context id): a device reset destroys the context, the
+// module is loaded again in the next one and the array may then sit elsewhere, so a new context
+// means a new lookup.  In host code the symbol names a host-side stand-in, never the device
+// memory, so kernels only ever receive this looked-up address.
 erc_status noalloc_scratch(void** out) {
   static std::mutex mu;
   static void* addr[64] = {};
+  static unsigned long long ctx_of[64] = {};
   int dev = 0;
   ERC_CUDA(cudaGetDevice(&dev));
   if (dev < 0 || dev >= 64) return set_error(ERC_ERR_CUDA, "device ordinal %d out of range", dev);
+  // 0 when no context is current yet (the lookup below makes the primary context current): the
+  // next call then looks up once more
+  const unsigned long long ctx = current_context_id();
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
+  if (!addr[dev] || ctx == 0 || ctx != ctx_of[dev]) {
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_probs_noalloc_scratch);
     if (e != cudaSuccess || !p)
       return set_error(ERC_ERR_CUDA, "cudaGetSymbolAddress(scratch) failed on device %d: %s",
                        dev, cudaGetErrorString(e));
     addr[dev] = p;
+    ctx_of[dev] = ctx;
   }
   *out = addr[dev];
   return ERC_OK;

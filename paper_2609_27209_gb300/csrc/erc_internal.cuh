@@ -42,6 +42,11 @@ inline cudaStream_t as_stream(erc_stream s) { return reinterpret_cast<cudaStream
 // SM count of the current device (cached per device).
 int sm_count();
 
+// Polls a bounded device-side wait makes before it gives up: `dflt` (the wait's own limit) unless
+// erc_set_wait_limit() set a process-wide override.  Read when work is enqueued (it is a kernel
+// argument, and part of the key of every cached graph that holds such a kernel).
+unsigned wait_limit(unsigned dflt);
+
 // process-wide count of kernels this library has launched (graph launches add the kernels they
 // contain); launches recorded while a graph is being captured are not counted
 void count_launches(long long k);
@@ -404,19 +409,29 @@ inline int grid_for(long long work_items, int items_per_block, int waves_blocks_
   return (int)g;
 }
 
+// A call's abort word (device): a bounded wait that gives up sets it, and every later kernel of
+// the same call that would consume the unfinished result returns at once when it is set; the host
+// reads it once the call's work has finished and reports ERC_ERR_TIMEOUT.
+__device__ __forceinline__ bool aborted(const unsigned* abort) {
+  return *reinterpret_cast<const volatile unsigned*>(abort) != 0u;
+}
+
 // ------------------------------------------------------------------------------------------------
 // internal entry points shared between translation units
 // ------------------------------------------------------------------------------------------------
 erc_status check_graph(const erc_graph* g);
 size_t scan_temp_bytes(int64_t n);
 // exclusive scan of int64 `in` (or of the 0/1 flags in `flags` when `in` is null) into `out`;
-// `total` (device, may be null) receives the sum.
+// `total` (device, may be null) receives the sum.  `abort` (device, required) is the call's abort
+// word: the scan does nothing when it is already set, and sets it when a bounded look-back wait
+// gives up (the output is then incomplete; every entry stays within [0, the true value]).
 erc_status exclusive_scan_i64(const int64_t* in, const uint8_t* flags, int64_t* out, int64_t n,
-                              int64_t* total, void* tmp, cudaStream_t s);
+                              int64_t* total, void* tmp, cudaStream_t s, unsigned* abort);
 size_t radix_sort_temp_bytes(int64_t n);
 // stable LSD radix sort of (key, value) pairs on the low `bits` key bits; the result is in
-// keys/vals (the *_alt buffers are scratch of the same size)
+// keys/vals (the *_alt buffers are scratch of the same size).  `abort` as for the scan: once it
+// is set no further pass runs and the result is undefined.
 erc_status radix_sort_pairs(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
-                            int64_t n, int bits, void* tmp, cudaStream_t s);
+                            int64_t n, int bits, void* tmp, cudaStream_t s, unsigned* abort);
 
 }  // namespace erc

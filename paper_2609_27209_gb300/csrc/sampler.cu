@@ -19,7 +19,7 @@ constexpr uint32_t SAMPLER_TAG = 0x53414D50u;
 struct SamplePlan {
   int64_t *W, *E, *draws, *npos, *epos, *totals;  // totals: [0] T [1] nodes [2] edges
   uint8_t *nmark, *emark;
-  unsigned* err;
+  unsigned* err;  // [0] a probability outside [0, 1]; [1] the abort word of the scans
   void* scan_tmp;
 };
 
@@ -183,13 +183,17 @@ extern "C" erc_status erc_sample_subgraph(const erc_graph* g, int32_t kind, cons
   k_fixed_weights<<<grid_for(count, ST), ST, 0, s>>>(prob, count, p.W, p.err);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
-  ERC_TRY(exclusive_scan_i64(p.W, nullptr, p.E, count, &p.totals[0], p.scan_tmp, s));
+  // the scans' prefixes are only ever below their true values when a bounded wait gives up, so
+  // every index derived from them stays in range; the host then reports the timeout
+  unsigned* abort = p.err + 1;
+  ERC_TRY(exclusive_scan_i64(p.W, nullptr, p.E, count, &p.totals[0], p.scan_tmp, s, abort));
   int64_t T = 0;
-  unsigned h_err = 0;
+  unsigned h_err[2] = {0, 0};
   ERC_CUDA(cudaMemcpyAsync(&T, p.totals, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
-  ERC_CUDA(cudaMemcpyAsync(&h_err, p.err, sizeof(unsigned), cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(h_err, p.err, 2 * sizeof(unsigned), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
-  if (h_err) return set_error(ERC_ERR_INVALID_ARG, "probabilities must lie in [0, 1]");
+  if (h_err[0]) return set_error(ERC_ERR_INVALID_ARG, "probabilities must lie in [0, 1]");
+  if (h_err[1]) return set_error(ERC_ERR_TIMEOUT, "a bounded wait in the sampler's scan ran out");
   if (T == 0) return set_error(ERC_ERR_INVALID_ARG, "every probability rounds to zero");
   const uint2 key = make_uint2((uint32_t)(seed & 0xffffffffu), (uint32_t)(seed >> 32));
   k_draw<<<grid_for(budget, ST), ST, 0, s>>>(p.E, count, p.totals, budget, key, first_draw,
@@ -205,19 +209,22 @@ extern "C" erc_status erc_sample_subgraph(const erc_graph* g, int32_t kind, cons
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
-  ERC_TRY(exclusive_scan_i64(nullptr, p.nmark, p.npos, g->n, &p.totals[1], p.scan_tmp, s));
+  ERC_TRY(exclusive_scan_i64(nullptr, p.nmark, p.npos, g->n, &p.totals[1], p.scan_tmp, s, abort));
   k_compact<<<grid_for(g->n, ST), ST, 0, s>>>(p.nmark, p.npos, g->n, nodes);
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   if (g->m > 0) {
-    ERC_TRY(exclusive_scan_i64(nullptr, p.emark, p.epos, g->m, &p.totals[2], p.scan_tmp, s));
+    ERC_TRY(exclusive_scan_i64(nullptr, p.emark, p.epos, g->m, &p.totals[2], p.scan_tmp, s,
+                               abort));
     k_compact<<<grid_for(g->m, ST), ST, 0, s>>>(p.emark, p.epos, g->m, edges);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
   }
   int64_t h_tot[3] = {0, 0, 0};
   ERC_CUDA(cudaMemcpyAsync(h_tot, p.totals, 3 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+  ERC_CUDA(cudaMemcpyAsync(h_err, p.err, 2 * sizeof(unsigned), cudaMemcpyDeviceToHost, s));
   ERC_CUDA(cudaStreamSynchronize(s));
+  if (h_err[1]) return set_error(ERC_ERR_TIMEOUT, "a bounded wait in the sampler's scans ran out");
   *n_out = (int32_t)h_tot[1];
   *m_out = g->m > 0 ? h_tot[2] : 0;
   return ERC_OK;

@@ -56,17 +56,23 @@ __device__ __forceinline__ int64_t block_exclusive_scan(int64_t v, int64_t* bloc
 // = aggregate, 2 = inclusive prefix); the tile's first warp walks back over its predecessors,
 // 32 at a time, until it meets an inclusive prefix.  Integer sums: the result does not depend on
 // the order in which tiles finish.  Inputs are non-negative and their total below 2^62.
+// Every poll of a predecessor's status is bounded: after `spin_limit` polls (or once another tile
+// has given up) the tile sets the call's abort word and takes the predecessor as an inclusive
+// prefix of zero, so its output stays within [0, the true prefix].  A block that starts after the
+// abort word is set takes no ticket and does nothing: no tile ever waits on a tile that no block
+// has claimed.
 constexpr unsigned LOOKBACK_SPINS = 1u << 22;
 
 template <class Load>
 __global__ void __launch_bounds__(SCAN_THREADS)
     k_scan_onepass(Load in, int64_t n, unsigned long long* status, unsigned* ticket, int64_t* out,
-                   int64_t* total, unsigned* timeout) {
+                   int64_t* total, unsigned* abort, unsigned spin_limit) {
   __shared__ int64_t tile[SCAN_TILE];
   __shared__ unsigned s_tile;
   __shared__ int64_t s_prefix;
-  if (threadIdx.x == 0) s_tile = atomicAdd(ticket, 1u);
+  if (threadIdx.x == 0) s_tile = aborted(abort) ? 0xffffffffu : atomicAdd(ticket, 1u);
   __syncthreads();
+  if (s_tile == 0xffffffffu) return;
   const int64_t t = s_tile;
   const int64_t base = t * SCAN_TILE;
 #pragma unroll
@@ -105,8 +111,8 @@ __global__ void __launch_bounds__(SCAN_THREADS)
         if (q >= 0) {
           unsigned spins = 0;
           while (((w = st[q]) & 3ull) == 0ull) {
-            if (++spins > LOOKBACK_SPINS) {  // bounded: record it and take zero
-              atomicOr(timeout, 1u);
+            if (++spins > spin_limit || aborted(abort)) {  // bounded: record it and take zero
+              atomicOr(abort, 1u);
               w = 2ull;
               break;
             }
@@ -148,10 +154,11 @@ __global__ void __launch_bounds__(SCAN_THREADS)
 
 inline int64_t scan_blocks(int64_t n) { return (n + SCAN_TILE - 1) / SCAN_TILE; }
 
-// tmp: [status: ntiles u64][ticket, timeout]
+// tmp: [status: ntiles u64][ticket]
 template <class Load>
 erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* tmp,
-                     cudaStream_t s) {
+                     cudaStream_t s, unsigned* abort) {
+  if (!abort) return set_error(ERC_ERR_INVALID_ARG, "internal: scan without an abort word");
   if (n <= 0) {
     if (total) ERC_CUDA(cudaMemsetAsync(total, 0, sizeof(int64_t), s));
     return ERC_OK;
@@ -160,8 +167,8 @@ erc_status scan_impl(Load in, int64_t n, int64_t* out, int64_t* total, int64_t* 
   unsigned long long* status = reinterpret_cast<unsigned long long*>(tmp);
   unsigned* ticket = reinterpret_cast<unsigned*>(status + nb);
   ERC_CUDA(cudaMemsetAsync(status, 0, (size_t)nb * sizeof(unsigned long long) + 8, s));
-  k_scan_onepass<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, status, ticket, out, total,
-                                                       ticket + 1);
+  k_scan_onepass<<<(unsigned)nb, SCAN_THREADS, 0, s>>>(in, n, status, ticket, out, total, abort,
+                                                       wait_limit(LOOKBACK_SPINS));
   count_launches(1);
   ERC_CUDA(cudaGetLastError());
   return ERC_OK;
@@ -183,9 +190,11 @@ inline int radix_bits(int64_t n) { return (n + RS_TILE - 1) / RS_TILE <= RS_WIDE
 
 template <int RB>
 __global__ void __launch_bounds__(RS_THREADS)
-    k_radix_hist(const uint64_t* keys, int64_t n, int shift, int64_t* counts, int64_t nb) {
+    k_radix_hist(const uint64_t* keys, int64_t n, int shift, int64_t* counts, int64_t nb,
+                 const unsigned* abort) {
   constexpr unsigned RADIX = 1u << RB;
   __shared__ unsigned hist[RADIX];
+  if (aborted(abort)) return;
   for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS) hist[d] = 0;
   __syncthreads();
   const int64_t base = (int64_t)blockIdx.x * RS_TILE;
@@ -203,10 +212,12 @@ template <int RB>
 __global__ void __launch_bounds__(RS_THREADS)
     k_radix_scatter(const uint64_t* __restrict__ keys, const uint32_t* __restrict__ vals,
                     uint64_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n,
-                    int shift, const int64_t* __restrict__ offsets, int64_t nb) {
+                    int shift, const int64_t* __restrict__ offsets, int64_t nb,
+                    const unsigned* abort) {
   constexpr unsigned RADIX = 1u << RB;
   __shared__ unsigned whist[RS_WARPS][RADIX];
   __shared__ int64_t boff[RADIX];
+  if (aborted(abort)) return;  // the offsets of an unfinished scan are not used
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (unsigned d = threadIdx.x; d < RADIX * RS_WARPS; d += RS_THREADS) (&whist[0][0])[d] = 0;
   for (unsigned d = threadIdx.x; d < RADIX; d += RS_THREADS)
@@ -257,7 +268,7 @@ __global__ void __launch_bounds__(RS_THREADS)
 
 template <int RB>
 erc_status radix_passes(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
-                        int64_t n, int bits, void* tmp, cudaStream_t s) {
+                        int64_t n, int bits, void* tmp, cudaStream_t s, unsigned* abort) {
   const int64_t nb = (n + RS_TILE - 1) / RS_TILE;
   const size_t cnt = (size_t)nb << RB;
   char* t = static_cast<char*>(tmp);
@@ -268,11 +279,12 @@ erc_status radix_passes(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint
   uint32_t *va = vals, *vb = vals_alt;
   int passes = 0;
   for (int shift = 0; shift < bits; shift += RB, ++passes) {
-    k_radix_hist<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, n, shift, counts, nb);
+    k_radix_hist<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, n, shift, counts, nb, abort);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
-    ERC_TRY(exclusive_scan_i64(counts, nullptr, offs, (int64_t)cnt, nullptr, scan_tmp, s));
-    k_radix_scatter<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, va, kb, vb, n, shift, offs, nb);
+    ERC_TRY(exclusive_scan_i64(counts, nullptr, offs, (int64_t)cnt, nullptr, scan_tmp, s, abort));
+    k_radix_scatter<RB><<<(unsigned)nb, RS_THREADS, 0, s>>>(ka, va, kb, vb, n, shift, offs, nb,
+                                                            abort);
     count_launches(1);
     ERC_CUDA(cudaGetLastError());
     uint64_t* tk = ka; ka = kb; kb = tk;
@@ -292,9 +304,9 @@ size_t scan_temp_bytes(int64_t n) {
 }
 
 erc_status exclusive_scan_i64(const int64_t* in, const uint8_t* flags, int64_t* out, int64_t n,
-                              int64_t* total, void* tmp, cudaStream_t s) {
-  if (in) return scan_impl(LoadI64{in}, n, out, total, static_cast<int64_t*>(tmp), s);
-  return scan_impl(LoadFlag{flags}, n, out, total, static_cast<int64_t*>(tmp), s);
+                              int64_t* total, void* tmp, cudaStream_t s, unsigned* abort) {
+  if (in) return scan_impl(LoadI64{in}, n, out, total, static_cast<int64_t*>(tmp), s, abort);
+  return scan_impl(LoadFlag{flags}, n, out, total, static_cast<int64_t*>(tmp), s, abort);
 }
 
 size_t radix_sort_temp_bytes(int64_t n) {
@@ -304,10 +316,11 @@ size_t radix_sort_temp_bytes(int64_t n) {
 }
 
 erc_status radix_sort_pairs(uint64_t* keys, uint32_t* vals, uint64_t* keys_alt, uint32_t* vals_alt,
-                            int64_t n, int bits, void* tmp, cudaStream_t s) {
+                            int64_t n, int bits, void* tmp, cudaStream_t s, unsigned* abort) {
   if (n <= 1) return ERC_OK;
-  if (radix_bits(n) == 10) return radix_passes<10>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s);
-  return radix_passes<8>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s);
+  if (radix_bits(n) == 10)
+    return radix_passes<10>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s, abort);
+  return radix_passes<8>(keys, vals, keys_alt, vals_alt, n, bits, tmp, s, abort);
 }
 
 }  // namespace erc

@@ -56,9 +56,13 @@ _SIGS = {
     "erc_version": (ctypes.c_char_p, []),
     "erc_last_error": (ctypes.c_char_p, []),
     "erc_kernel_launches": (ctypes.c_uint64, []),
+    "erc_set_wait_limit": (None, [ctypes.c_uint32]),
     "erc_build_laplacian_workspace_size": (_sz, [_i32, _i64]),
     "erc_build_laplacian": (_i32, [_i32, _c_p, _c_p, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, ctypes.POINTER(_i64), _c_p, _sz, _c_p]),
+    "erc_build_laplacian_ex": (_i32, [_i32, _c_p, _c_p, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p,
+                                      _c_p, _c_p, _c_p, _c_p, ctypes.POINTER(_i64),
+                                      ctypes.POINTER(_i32), _c_p, _sz, _c_p]),
     "erc_jl_rhs": (_i32, [ctypes.POINTER(ErcGraphC), _u64, _i32, _i32, _i32, _c_p, _i32, _c_p]),
     "erc_batched_cg_workspace_size": (_sz, [_i32, _i32]),
     "erc_batched_cg": (_i32, [ctypes.POINTER(ErcGraphC), _f32, _c_p, _c_p, _i32, _i32, _f32,
@@ -151,6 +155,11 @@ def erc_kernel_launches():
     return int(lib().erc_kernel_launches())
 
 
+def erc_set_wait_limit(polls):
+    """Polls every bounded device-side wait makes before giving up (0 restores the defaults)."""
+    lib().erc_set_wait_limit(int(polls))
+
+
 @dataclass
 class Graph:
     """Tensors of a graph built by erc_build_laplacian plus the matching C struct."""
@@ -193,14 +202,15 @@ def erc_build_laplacian(n, src, dst, w=None, dup_policy=ERC_DUP_SUM):
     ew = torch.empty(cap1, dtype=torch.float32, device=dev)
     ws = _workspace(lib().erc_build_laplacian_workspace_size(n, m_in), dev)
     m = _i64(0)
-    _check(lib().erc_build_laplacian(n, _ptr(src), _ptr(dst), _ptr(w), m_in, dup_policy,
-                                     _ptr(row_ptr), _ptr(col), _ptr(val), _ptr(deg),
-                                     _ptr(csr_eid), _ptr(eu), _ptr(ev), _ptr(ew),
-                                     ctypes.byref(m), _ptr(ws), ws.numel(), _stream()))
+    unit = _i32(0)
+    _check(lib().erc_build_laplacian_ex(n, _ptr(src), _ptr(dst), _ptr(w), m_in, dup_policy,
+                                        _ptr(row_ptr), _ptr(col), _ptr(val), _ptr(deg),
+                                        _ptr(csr_eid), _ptr(eu), _ptr(ev), _ptr(ew),
+                                        ctypes.byref(m), ctypes.byref(unit), _ptr(ws), ws.numel(),
+                                        _stream()))
     m = m.value
-    unit = bool(w is None and (m == 0 or bool((ew[:m] == 1).all())))
     return Graph(n, m, row_ptr, col[:2 * m], val[:2 * m], deg, csr_eid[:2 * m], eu[:m], ev[:m],
-                 ew[:m], unit)
+                 ew[:m], bool(unit.value))
 
 
 def padded_ld(kc):

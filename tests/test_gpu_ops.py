@@ -26,6 +26,22 @@ def test_build_multigraph_bit_exact(seed, policy, weighted):
     assert_graph_equal(g, ref)
 
 
+@pytest.mark.parametrize("policy", [0, 1])
+def test_build_reports_unit_weights(policy):
+    """erc_build_laplacian_ex's unit-weight flag: 1 exactly when no weights were given and every
+    merged weight is 1 (duplicates summed under ERC_DUP_SUM give 2; ERC_DUP_FIRST keeps 1)."""
+    n, src, dst, _ = synth.random_connected(300, 900, seed=5)
+    g = erc.erc_build_laplacian(n, to_dev(src), to_dev(dst), None, policy)
+    assert g.unit_weights and bool((g.ew == 1).all())
+    g = erc.erc_build_laplacian(n, to_dev(src), to_dev(dst),
+                                to_dev(np.ones(src.size, np.float32)), policy)
+    assert not g.unit_weights  # weights were given: the graph keeps its weight arrays
+    dup_src, dup_dst = np.concatenate([src, dst[:5]]), np.concatenate([dst, src[:5]])
+    g = erc.erc_build_laplacian(n, to_dev(dup_src), to_dev(dup_dst), None, policy)
+    assert g.unit_weights == (policy == 1)
+    assert bool((g.ew == 1).all()) == (policy == 1)
+
+
 @pytest.mark.parametrize("name", ["ring_chords_n2000", "sbm_n20000"])
 def test_build_workload_bit_exact(name):
     g, ref = build_both(*synth.make_graph(name))

@@ -57,3 +57,26 @@ def test_noalloc_rejects_graphs_beyond_its_limit():
                                               erc._ptr(out), erc._ptr(out), erc._stream())
     assert st == erc.ERC_ERR_CAPACITY
     assert b"at most 4000000 nodes" in erc.lib().erc_last_error()
+
+
+def test_noalloc_call_allocates_no_device_memory():
+    """With its outputs preallocated, a warmed-up call leaves the device's free memory and the
+    torch allocator's reservation unchanged: the scratch is the library's static array."""
+    n, src, dst, w = synth.random_connected(50_000, 200_000, seed=23, weighted=True)
+    g = erc.erc_build_laplacian(n, _dev(src), _dev(dst), _dev(w))
+    kappa = _dev(synth.random_normal(g.m, seed=33, scale=1.5))
+    out = (torch.empty(g.n, dtype=torch.float32, device="cuda:0"),
+           torch.empty(g.m, dtype=torch.float32, device="cuda:0"))
+    erc.erc_sampling_probs_noalloc(g, kappa, 1e-8, out=out)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    reserved0 = torch.cuda.memory_reserved()
+    for _ in range(3):
+        erc.erc_sampling_probs_noalloc(g, kappa, 1e-8, out=out)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0
+    assert torch.cuda.memory_reserved() == reserved0
+    ref_n, ref_e = erc.erc_sampling_probs(g, kappa, 1e-8)
+    np.testing.assert_allclose(out[0].cpu().numpy(), ref_n.cpu().numpy(), rtol=1e-6, atol=1e-12)
+    np.testing.assert_allclose(out[1].cpu().numpy(), ref_e.cpu().numpy(), rtol=1e-6)
