@@ -4,9 +4,11 @@
 One step = the whole path on one synthetic graph with its inputs resident in HBM: Laplacian build,
 then for every batch of projection columns the Philox right-hand sides, the column-wise CG solve
 and the edge-resistance accumulation, then curvature (Eq. 2) and the sampling probabilities
-(Eq. 7-8).  The metric is curvature edges per second (m / step time); the JSON line also carries
-the end-to-end number through the host-memory C-ABI call, the roofline of the dominant kernel
-(the L_eps P gather), the CPU oracle as a reported baseline, clocks and the kernel-launch count.
+(Eq. 7-8).  The metric is curvature edges per second (m / step time).  The default workload is the
+largest: the 2.45M-node, 64.3M-edge power-law graph at K = 1024 in batches of 128 columns (its
+smaller K = 64 and 256 are reported under "k_sweep").  The JSON line also carries the end-to-end
+number through the host-memory C-ABI call, the roofline of the dominant kernel, the CPU oracle as
+a reported baseline, clocks and the kernel-launch count.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config NAME]
 Under torchrun (N > 1) every rank owns K projection columns of a K*N projection (weak scaling)
@@ -29,7 +31,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "ERC-LG curvature edges/s end-to-end; CG SpMM HBM GB/s vs GB300 peak"
-DEFAULT_CONFIG = "sbm_n20000"
+DEFAULT_CONFIG = "chung_lu_n2449029_g2.3"
 
 
 def parse():
@@ -39,8 +41,11 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
-    ap.add_argument("--K", type=int, default=None, help="projection dimension (per rank)")
+    ap.add_argument("--K", type=int, default=None,
+                    help="projection dimension (per rank; default: the workload's largest)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the workload's other projection dimensions")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--spmm-reps", type=int, default=50)
     ap.add_argument("--precond", choices=["none", "jacobi"], default="none",
@@ -147,35 +152,91 @@ def spmm_algorithmic_bytes(n, m, kc, weighted):
 
 
 # ------------------------------------------------------------------------------------ oracle leg
+# The float64 oracle (oracle/erc_oracle.py, as it stands) timed on the host cores on a bounded
+# sample of the workload.  A run costs build + K x (one column's right-hand side, CG solve and
+# edge distances: the K systems are independent and cost alike) + the curvature/probability tail.
+# Up to CAPPED_EDGES edges the sample solves whole columns; beyond that one column's solve takes
+# minutes, so the sample runs CAP_ITERS CG iterations of one column and scales them to the
+# column's iteration count.
+CAPPED_EDGES = 10_000_000
+CAP_ITERS = 20
+
+
 def _oracle_solver(precond):
     from oracle import erc_oracle as O
     return O.batched_pcg if precond == "jacobi" else O.batched_cg
 
 
-def oracle_sample(name, K, cols, precond="none"):
-    """Time the CPU oracle on the full graph with `cols` of the K projection columns and
-    extrapolate the column-proportional part to K.  Returns (edges/s, seconds, description)."""
-    import numpy as np
+class OracleRun:
+    """The oracle's graph of one workload, with the seconds its build took."""
 
-    from oracle import erc_oracle as O
-    from paper_2609_27209_gb300 import synth
+    def __init__(self, name, precond="none", graph=None):
+        from oracle import erc_oracle as O
+        from paper_2609_27209_gb300 import synth
 
-    wl = synth.WORKLOADS[name]
-    n, src, dst, w = synth.make_graph(name)
+        self.name, self.precond = name, precond
+        self.wl = synth.WORKLOADS[name]
+        self.seed = synth.JL_SEED
+        n, src, dst, w = synth.make_graph(name) if graph is None else graph
+        t0 = time.perf_counter()
+        self.g = O.build_laplacian(n, src, dst, w)
+        self.t_build = time.perf_counter() - t0
+        self.n, self.m = n, self.g["m"]
+        self.capped = self.m > CAPPED_EDGES
+
+    def columns(self, K, c0, cols, max_iter=20000):
+        """(t_rhs, t_cg, t_edge, iterations, R) of columns [c0, c0 + cols) of the K projection."""
+        from oracle import erc_oracle as O
+
+        t0 = time.perf_counter()
+        Y = O.jl_rhs(self.g, self.seed, K, c0, cols)
+        t1 = time.perf_counter()
+        X, it, _, _ = _oracle_solver(self.precond)(self.g, self.wl.eps, Y, self.wl.tol, max_iter)
+        t2 = time.perf_counter()
+        R = O.edge_resistance(self.g, X)
+        t3 = time.perf_counter()
+        return t1 - t0, t2 - t1, t3 - t2, it, R
+
+    def tail(self, R):
+        from oracle import erc_oracle as O
+
+        t0 = time.perf_counter()
+        _, kappa = O.curvature(self.g, R)
+        O.sampling_probs(self.g, kappa)
+        return time.perf_counter() - t0
+
+    def column_iterations(self, K):
+        """CG iterations of column 0 solved to the tolerance (the capped samples' scale)."""
+        return int(self.columns(K, 0, 1)[3][0])
+
+
+def oracle_sample(run, K, cols):
+    """Whole columns: the full graph with `cols` of the K columns, the column work scaled to K.
+    Returns (edges/s, seconds sampled, description, estimated seconds of the whole run)."""
     t0 = time.perf_counter()
-    g = O.build_laplacian(n, src, dst, w)
-    t1 = time.perf_counter()
-    Y = O.jl_rhs(g, synth.JL_SEED, K, 0, cols)
-    X, it, _, _ = _oracle_solver(precond)(g, wl.eps, Y, wl.tol)
-    R = O.edge_resistance(g, X)
-    t2 = time.perf_counter()
-    p, kappa = O.curvature(g, R * (K / cols))
-    O.sampling_probs(g, kappa)
-    t3 = time.perf_counter()
-    est = (t1 - t0) + (t2 - t1) * (K / cols) + (t3 - t2)
-    desc = (f"full graph (n={n}, m={g['m']}), {cols} of {K} projection columns; build and "
-            f"curvature/probability tail timed once, the per-column solve scaled by {K}/{cols}")
-    return g["m"] / est, t3 - t0, desc, est
+    tr, tc, te, _, R = run.columns(K, 0, cols)
+    t_tail = run.tail(R * (K / cols))
+    est = run.t_build + (tr + tc + te) * (K / cols) + t_tail
+    desc = (f"full graph (n={run.n}, m={run.m}), {cols} of {K} projection columns solved to the "
+            f"tolerance; build ({run.t_build:.1f} s) and curvature/probability tail timed once, "
+            f"the column work scaled by {K}/{cols}")
+    return run.m / est, time.perf_counter() - t0 + run.t_build, desc, est
+
+
+def oracle_sample_capped(run, K, T, t_tail=None, cap=CAP_ITERS):
+    """One column with its CG capped at `cap` iterations, scaled to T iterations per column and to
+    K columns.  Returns (edges/s, seconds sampled, description, estimated seconds)."""
+    t0 = time.perf_counter()
+    tr, tc, te, it, R = run.columns(K, 0, 1, max_iter=cap)
+    done = max(1, int(it[0]))
+    if t_tail is None:
+        t_tail = run.tail(R * K)
+    est = run.t_build + K * (tr + tc * (T / done) + te) + t_tail
+    desc = (f"full graph (n={run.n}, m={run.m}); build ({run.t_build:.1f} s) and "
+            f"curvature/probability tail ({t_tail:.1f} s) timed once; one column's right-hand "
+            f"side, {done} CG iterations and edge distances timed, the iterations scaled to "
+            f"{T:.1f} per column and the column to {K} columns")
+    return run.m / est, time.perf_counter() - t0, desc, est
 
 
 def cpu_cores_used():
@@ -205,18 +266,13 @@ def _oracle_columns(task):
     return O.edge_resistance(g, X)
 
 
-def oracle_sample_all_cores(name, K, cols, procs, precond="none"):
+def oracle_sample_all_cores(run, K, cols, procs):
     """The same sample as oracle_sample with the `cols` columns split over `procs` processes
     (spawn context, one BLAS thread each, warmed up before timing); the build and the
-    curvature/probability tail are not parallel and are timed once on one core."""
+    curvature/probability tail are not parallel and are counted once on one core."""
     import multiprocessing as mp
 
     from oracle import erc_oracle as O
-    from paper_2609_27209_gb300 import synth
-    n, src, dst, w = synth.make_graph(name)
-    t0 = time.perf_counter()
-    g = O.build_laplacian(n, src, dst, w)
-    t_build = time.perf_counter() - t0
     saved = {k: os.environ.get(k) for k in _THREAD_VARS}
     for k in _THREAD_VARS:
         os.environ[k] = "1"
@@ -224,7 +280,7 @@ def oracle_sample_all_cores(name, K, cols, procs, precond="none"):
         with mp.get_context("spawn").Pool(procs) as pool:
             pool.map(_oracle_warm, range(4 * procs), chunksize=1)
             bounds = [(cols * i // procs, cols * (i + 1) // procs) for i in range(procs)]
-            tasks = [(name, K, a, b - a, g, precond) for a, b in bounds if b > a]
+            tasks = [(run.name, K, a, b - a, run.g, run.precond) for a, b in bounds if b > a]
             t0 = time.perf_counter()
             parts = pool.map(_oracle_columns, tasks, chunksize=1)
             t_cols = time.perf_counter() - t0
@@ -236,30 +292,53 @@ def oracle_sample_all_cores(name, K, cols, procs, precond="none"):
                 os.environ[k] = v
     R = sum(parts)
     t0 = time.perf_counter()
-    _, kappa = O.curvature(g, R * (K / cols))
-    O.sampling_probs(g, kappa)
+    _, kappa = O.curvature(run.g, R * (K / cols))
+    O.sampling_probs(run.g, kappa)
     t_tail = time.perf_counter() - t0
-    est = t_build + t_cols * (K / cols) + t_tail
-    desc = (f"full graph (n={n}, m={g['m']}), {cols} of {K} projection columns split over "
+    est = run.t_build + t_cols * (K / cols) + t_tail
+    desc = (f"full graph (n={run.n}, m={run.m}), {cols} of {K} projection columns split over "
             f"{len(tasks)} processes; build and curvature/probability tail on one core, the "
             f"column work scaled by {K}/{cols}")
-    return g["m"] / est, desc
+    return run.m / est, desc
 
 
 # ------------------------------------------------------------------------------------ main legs
+def workload_K(args, wl):
+    """The projection dimension of the run: --K, else the workload's largest."""
+    return args.K or max(wl.K)
+
+
 def run_reference(args, world, rank):
+    """The float64 oracle on the host cores as the reference arm: every step is a bounded sample
+    of the workload (see the oracle leg); rank 0 alone runs it."""
     from paper_2609_27209_gb300 import synth
 
     wl = synth.WORKLOADS[args.config]
-    K = args.K or wl.K[0]
-    cols = max(4, K // 8)
+    K = workload_K(args, wl)
     if rank != 0:
         return
+    run = OracleRun(args.config, args.precond)
+    if run.capped:
+        # the iterations a column needs, from one full oracle solve (column 0), and the tail,
+        # both once; every step then times one capped column
+        T = run.column_iterations(K)
+        _, _, _, _, R = run.columns(K, 0, 1, max_iter=CAP_ITERS)
+        t_tail = run.tail(R * K)
+
+        def sample():
+            v, secs, desc, est = oracle_sample_capped(run, K, T, t_tail)
+            return v, secs, desc + f" (from a full oracle solve of column 0: {T} iterations)", est
+    else:
+        cols = min(K, max(4, K // 8))
+
+        def sample():
+            return oracle_sample(run, K, cols)
     for _ in range(args.warmup):
-        oracle_sample(args.config, K, cols, args.precond)
+        sample()
     vals, ests = [], []
+    desc = ""
     for _ in range(args.steps):
-        v, _, desc, est = oracle_sample(args.config, K, cols, args.precond)
+        v, _, desc, est = sample()
         vals.append(v)
         ests.append(est)
     value = len(vals) / sum(1.0 / v for v in vals)  # harmonic mean = m / mean time
@@ -267,13 +346,31 @@ def run_reference(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * statistics.mean(ests), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.config, "K": K, "kc": wl.kc, "eps": wl.eps,
+            "config": {"workload": args.config, "K": K, "kc": min(wl.kc, K), "eps": wl.eps,
                        "tol": wl.tol, "precond": args.precond},
             "cpu_baseline": {"value": value, "unit": "edges/s", "cores": cpu_cores_used(),
                              "kind": "oracle", "sample": desc},
             "e2e": {"value": value, "unit": "edges/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def _timed_steps(step, n_steps, flush, stream):
+    """CUDA-event time (ms) of each of n_steps calls of step(), L2 flushed before each."""
+    import torch
+
+    times = []
+    res = None
+    for _ in range(n_steps):
+        flush.fill_(1)  # evict L2 between timed steps (outside the timed interval)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        res = step()
+        b.record(stream)
+        b.synchronize()
+        times.append(a.elapsed_time(b))
+    return times, res
 
 
 def run_ours(args, world, rank, local_rank):
@@ -287,17 +384,18 @@ def run_ours(args, world, rank, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     wl = synth.WORKLOADS[args.config]
-    K = args.K or wl.K[0]
+    K = workload_K(args, wl)
     kc = min(wl.kc, K)
-    n, src, dst, w = synth.make_graph(args.config)
+    graph = synth.make_graph(args.config)
+    n, src, dst, w = graph
     m_in = src.size
-    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED,
-                     precond=erc.ERC_PRECOND_JACOBI if args.precond == "jacobi"
-                     else erc.ERC_PRECOND_NONE)
+    precond = erc.ERC_PRECOND_JACOBI if args.precond == "jacobi" else erc.ERC_PRECOND_NONE
+    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED, precond=precond)
     src_d = torch.from_numpy(src).to(dev)
     dst_d = torch.from_numpy(dst).to(dev)
     w_d = None if w is None else torch.from_numpy(w).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB of L2
+    stream = torch.cuda.current_stream()
 
     mem = None
     if world == 1:
@@ -325,23 +423,13 @@ def run_ours(args, world, rank, local_rank):
         res = step()
     torch.cuda.synchronize()
     m = int(res["m"])
-    stream = torch.cuda.current_stream()
     sampler = ClockSampler(local_rank)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     launches0 = erc.erc_kernel_launches()
     sampler.start()
-    times = []
-    for _ in range(args.steps):
-        flush.fill_(1)  # evict L2 between timed steps (outside the timed interval)
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        res = step()
-        b.record(stream)
-        b.synchronize()
-        times.append(a.elapsed_time(b))
+    times, res = _timed_steps(step, args.steps, flush, stream)
     torch.cuda.synchronize()
     clocks = sampler.stop()
     launches = erc.erc_kernel_launches() - launches0
@@ -355,6 +443,9 @@ def run_ours(args, world, rank, local_rank):
     value = world * m / (ms_max / 1000.0)
     iters = res.get("iters")
     it = iters.float() if iters is not None else None
+    slow = ms_max > 2000.0  # steps of seconds: fewer repetitions of the extra measurements
+    if world == 1:
+        del ws, out
 
     # ---- end to end through the host-memory C-ABI call (copies inside the timed region)
     e2e = None
@@ -364,10 +455,10 @@ def run_ours(args, world, rank, local_rank):
         w_h = None if w is None else torch.from_numpy(w).pin_memory()
         hws = erc.erc_run_host_workspace(n, m_in, prm, dev)
         hout = erc._run_outputs(n, m_in, K, None, pin=True)
-        for _ in range(2):
+        for _ in range(1 if slow else 2):
             erc.erc_run_host(n, src_h, dst_h, w_h, prm, ws=hws, out=hout)
         et = []
-        for _ in range(max(3, args.steps // 2)):
+        for _ in range(3 if slow else max(3, args.steps // 2)):
             flush.fill_(1)
             torch.cuda.synchronize()
             t0 = time.perf_counter()
@@ -377,19 +468,36 @@ def run_ours(args, world, rank, local_rank):
         h2d = m_in * 4 * (2 if w is None else 3)
         d2h = 5 * 4 * m + 2 * 4 * n + 2 * 4 * K
         e2e = {"value": m / statistics.mean(et), "unit": "edges/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": 1000 * statistics.mean(et)}
+               "d2h_bytes_per_step": d2h, "ms_per_step": 1000 * statistics.mean(et),
+               "repetitions": len(et)}
+        del hws, hout
+
+    # ---- the workload's other projection dimensions (its K sweep), the same path and batches
+    sweep = None
+    if world == 1 and not args.no_sweep and len(wl.K) > 1:
+        sweep = []
+        for Ks in wl.K:
+            if Ks == K:
+                continue
+            p2 = erc.Params(K=Ks, kc=min(wl.kc, Ks), eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED,
+                            precond=precond)
+            ws2 = erc.erc_run_workspace(n, m_in, p2, dev)
+            out2 = erc._run_outputs(n, m_in, Ks, dev)
+            st2 = lambda: erc.erc_run(n, src_d, dst_d, w_d, p2, ws=ws2, out=out2)
+            st2()
+            t2, r2 = _timed_steps(st2, 3, flush, stream)
+            sweep.append({"K": Ks, "kc": p2.kc, "ms_per_step": statistics.mean(t2),
+                          "value": m / (statistics.mean(t2) / 1000.0), "status": r2["status"],
+                          "cg_iters_mean": float(r2["iters"].float().mean())})
+            del ws2, out2
+        torch.cuda.empty_cache()
 
     # ---- roofline of the dominant kernel.  On graphs whose r and Ap blocks fit in shared memory
-    # the whole CG solve is one launch (k_cg_cluster over column groups, else k_cg_resident): its
-    # duration comes from CUDA events the library records around it on its stream.  Otherwise the operator k_spmm dominates and is
-    # timed alone, back to back as inside the CG loop.  Either way the operator alone is also
-    # reported under "spmm".
-    roof = None
-    spmm = None
-    cusparse = None
-    sampler = None
-    cpu_all = None
-    variants = None
+    # the whole CG solve is one launch (k_cg_cluster over column groups, else k_cg_resident),
+    # timed by CUDA events the library records around it on its stream; its bytes stay in L2.
+    # Otherwise the operator k_spmm dominates (HBM: P exceeds L2) and is timed alone, back to back
+    # as inside the CG loop.  The operator alone is always reported under "spmm".
+    roof = spmm = cusparse = samp = cpu_all = variants = None
     if rank == 0:
         g = erc.erc_build_laplacian(n, src_d, dst_d, w_d)
         P = erc.erc_jl_rhs(g, synth.JL_SEED, K, 0, kc)
@@ -398,9 +506,14 @@ def run_ours(args, world, rank, local_rank):
         op_bytes = spmm_algorithmic_bytes(n, g.m, kc, weighted)
         erc.erc_laplacian_apply_timed(g, prm.eps, P, kc, reps=5)
         t_spmm = erc.erc_laplacian_apply_timed(g, prm.eps, P, kc, reps=args.spmm_reps) * 1e-6
+        traffic = spmm_traffic(args.config)
         spmm = {"kernel": "k_spmm (L_eps P + p.Ap)", "launch_us": t_spmm * 1e6,
                 "algorithmic_bytes": op_bytes, "achieved": op_bytes / t_spmm / 1e9,
-                "frac": op_bytes / t_spmm / 1e9 / peak, "traffic": spmm_traffic(args.config)}
+                "frac": op_bytes / t_spmm / 1e9 / peak, "traffic": traffic,
+                "gathered_row_bytes": 4 * 2 * g.m * kc}
+        if traffic:
+            spmm["dram_achieved"] = traffic / t_spmm / 1e9
+            spmm["dram_frac"] = spmm["dram_achieved"] / peak
         # library comparison point (run only): cuSPARSE SpMM of the adjacency, A P, through
         # torch's CSR x dense product, timed with events on the current stream
         vals = g.val if not g.unit_weights else torch.ones(2 * g.m, device=dev)
@@ -409,23 +522,24 @@ def run_ours(args, world, rank, local_rank):
             A = torch.sparse_csr_tensor(g.row_ptr, g.col.long(), vals, size=(n, n))
         for _ in range(3):
             A @ P
+        reps = 10 if slow else args.spmm_reps
         ca, cb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ca.record()
-        for _ in range(args.spmm_reps):
+        for _ in range(reps):
             A @ P
         cb.record()
         cb.synchronize()
-        t_cs = ca.elapsed_time(cb) / 1e3 / args.spmm_reps
+        t_cs = ca.elapsed_time(cb) / 1e3 / reps
         cusparse = {"kernel": "cuSPARSE SpMM A P (torch sparse CSR @ dense), run only",
                     "launch_us": t_cs * 1e6, "achieved": op_bytes / t_cs / 1e9,
                     "frac": op_bytes / t_cs / 1e9 / peak}
-        del A
+        del A, vals
         # the curvature-guided subgraph samplers on this run's probabilities (§3.2), one call
         # each (node budget n/10, edge budget m/10); each call synchronises to return its sizes
         if res.get("prob_node") is not None and res.get("prob_edge") is not None:
-            sampler = {"node_budget": max(1, n // 10), "edge_budget": max(1, g.m // 10)}
-            runs = [(erc.ERC_SAMPLE_NODES, "node", res["prob_node"], sampler["node_budget"]),
-                    (erc.ERC_SAMPLE_EDGES, "edge", res["prob_edge"], sampler["edge_budget"])]
+            samp = {"node_budget": max(1, n // 10), "edge_budget": max(1, g.m // 10)}
+            runs = [(erc.ERC_SAMPLE_NODES, "node", res["prob_node"], samp["node_budget"]),
+                    (erc.ERC_SAMPLE_EDGES, "edge", res["prob_edge"], samp["edge_budget"])]
             for kind, key, prob, b in runs:
                 sws = erc._workspace(erc.lib().erc_sample_workspace_size(n, g.m, b), dev)
                 erc.erc_sample_subgraph(g, kind, prob, b, 1, ws=sws)
@@ -434,8 +548,9 @@ def run_ours(args, world, rank, local_rank):
                 for r in range(5):
                     nodes_s, edges_s = erc.erc_sample_subgraph(g, kind, prob, b, 1, b * r, ws=sws)
                 torch.cuda.synchronize()
-                sampler[key + "_subgraph_us"] = (time.perf_counter() - t0) / 5 * 1e6
-                sampler[key + "_subgraph_size"] = [int(nodes_s.numel()), int(edges_s.numel())]
+                samp[key + "_subgraph_us"] = (time.perf_counter() - t0) / 5 * 1e6
+                samp[key + "_subgraph_size"] = [int(nodes_s.numel()), int(edges_s.numel())]
+                del sws
         erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)  # warm
         _, it_cg, _, _, solve_us, path = erc.erc_batched_cg_timed(g, prm.eps, P, kc, prm.tol)
         # the optional Jacobi-preconditioned solve of the same batch (not the paper's solver)
@@ -452,40 +567,57 @@ def run_ours(args, world, rank, local_rank):
         if pc:
             it_cg, solve_us, path = it_pc, pcg_us, pcg_path
         if path in (1, 2):
-            T = int(it_cg.max().item())
-            # T iterations, plus the launch's own initialisation (read Y; write P, X) and, in the
-            # resident kernel, the true residual (one operator application on X, Y read)
-            algo = T * (op_bytes + UPDATE_BYTES_PER_ELEM * n * kc) + 12 * n * kc
+            # bytes the solve must move: the CSR once per iteration while any column is active,
+            # per column and iteration it runs P once, Ap once and the update's 7 vector passes
+            # (a converged column is neither gathered nor updated), plus the launch's own
+            # initialisation (read Y; write P, X) and, in the resident kernel, the true residual
+            its = it_cg.double()
+            T = int(its.max().item())
+            csr = op_bytes - 2 * 4 * n * kc
+            algo = T * csr + float(its.sum().item()) * (8 + UPDATE_BYTES_PER_ELEM) * n
+            algo += 12 * n * kc
             if path == 1:
                 algo += op_bytes + 4 * n * kc
             ach = algo / (solve_us * 1e-6) / 1e9
             kname = "k_cg_cluster" if path == 2 else "k_cg_resident"
-            roof = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+            roof = {"bound": "l2", "achieved": ach, "peak": peak, "unit": "GB/s",
                     "frac": ach / peak,
                     "traffic": None if pc else _traffic(kname[2:], args.config),
                     "kernel": f"{kname}{' (Jacobi)' if pc else ''} (one launch = whole CG solve "
-                              "of a batch)",
-                    "iterations": T, "algorithmic_bytes": algo, "launch_us": solve_us,
-                    "peak_source": src_kind}
+                              "of a batch; its working set stays in L2, so frac is an effective "
+                              "rate against the HBM peak)",
+                    "iterations": T, "column_iterations": float(its.sum().item()),
+                    "algorithmic_bytes": algo, "launch_us": solve_us, "peak_source": src_kind}
         else:
             roof = {"bound": "hbm", "achieved": spmm["achieved"], "peak": peak, "unit": "GB/s",
                     "frac": spmm["frac"], "traffic": spmm["traffic"], "kernel": spmm["kernel"],
                     "algorithmic_bytes": op_bytes, "launch_us": t_spmm * 1e6,
-                    "peak_source": src_kind}
+                    "peak_source": src_kind, "gathered_row_bytes": spmm["gathered_row_bytes"]}
+            if traffic:
+                roof["dram_achieved"] = spmm["dram_achieved"]
+                roof["dram_frac"] = spmm["dram_frac"]
+        del g, P
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # size the sample to roughly 15 s of CPU work from a 4-column probe
-        _, _, _, est4 = oracle_sample(args.config, K, 4, args.precond)
-        per_col = est4 / K  # the probe's estimate is for all K columns
-        cols = int(min(K, max(4, (15.0 / max(per_col, 1e-9)) // 4 * 4)))
-        v, secs, desc, est = oracle_sample(args.config, K, cols, args.precond)
-        procs = max(1, min(os.cpu_count() or 1, cols))
-        va, desc_all = oracle_sample_all_cores(args.config, K, cols, procs, args.precond)
-        cpu_all = {"value": va, "unit": "edges/s", "cores": procs, "kind": "oracle",
-                   "sample": desc_all}
+        run = OracleRun(args.config, args.precond, graph=graph)
+        if run.capped:
+            T_gpu = float(it.mean())  # the solver's iterations per column on this workload
+            v, secs, desc, _ = oracle_sample_capped(run, K, T_gpu)
+            desc += " (the iteration count is the GPU solve's mean)"
+        else:
+            # size the sample to roughly 15 s of CPU work from a 4-column probe
+            _, _, _, est4 = oracle_sample(run, K, min(K, 4))
+            per_col = (est4 - run.t_build) / K
+            cols = int(min(K, max(4, (15.0 / max(per_col, 1e-9)) // 4 * 4)))
+            v, secs, desc, _ = oracle_sample(run, K, cols)
+            procs = max(1, min(os.cpu_count() or 1, cols))
+            va, desc_all = oracle_sample_all_cores(run, K, cols, procs)
+            cpu_all = {"value": va, "unit": "edges/s", "cores": procs, "kind": "oracle",
+                       "sample": desc_all}
         cpu = {"value": v, "unit": "edges/s", "cores": cpu_cores_used(), "kind": "oracle",
                "sample": desc, "seconds": secs}
+        del run
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "edges/s", "n_gpus": world,
@@ -496,8 +628,8 @@ def run_ours(args, world, rank, local_rank):
                            "eps": wl.eps, "tol": wl.tol, "precond": args.precond,
                            "l2": "flushed (256 MiB write) before every timed step",
                            "parallelism": f"projection columns over {world} rank(s)"},
-                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": sampler,
-                "solver_variants": variants, "cpu_baseline": cpu,
+                "roofline": roof, "spmm": spmm, "cusparse_spmm": cusparse, "sampler": samp,
+                "solver_variants": variants, "k_sweep": sweep, "cpu_baseline": cpu,
                 "cpu_baseline_all_cores": cpu_all,
                 "e2e": e2e, "gpu_launches": launches, "device_memory_bytes": mem,
                 "clocks": clocks,

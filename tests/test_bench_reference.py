@@ -58,3 +58,25 @@ def test_operator_algorithmic_bytes():
     unweighted = 4 * 2 * m + 8 * (n + 1) + 2 * 4 * n * kc
     assert bench.spmm_algorithmic_bytes(n, m, kc, False) == unweighted
     assert bench.spmm_algorithmic_bytes(n, m, kc, True) == unweighted + 4 * 2 * m
+
+
+def test_capped_oracle_sample_keeps_the_contract(monkeypatch, capsys):
+    """The sample used on graphs of more than CAPPED_EDGES edges (one column's CG capped, scaled
+    to the column's iteration count), exercised on the 2k-node workload."""
+    import argparse
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    monkeypatch.setattr(bench, "CAPPED_EDGES", 0)
+    args = argparse.Namespace(config="ring_chords_n2000", K=None, steps=2, warmup=1, gpus=1,
+                              precond="none")
+    bench.run_reference(args, 1, 0)
+    d = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["config"]["K"] == 64
+    assert "CG iterations" in d["cpu_baseline"]["sample"]
+    assert "full oracle solve of column 0" in d["cpu_baseline"]["sample"]
+    run = bench.OracleRun("ring_chords_n2000")
+    T = run.column_iterations(64)
+    v, _, desc, est = bench.oracle_sample_capped(run, 64, T, cap=5)
+    assert v > 0 and est > run.t_build and "5 CG iterations" in desc
