@@ -302,6 +302,8 @@ __global__ void __launch_bounds__(T) k_cg_init(VecArgs a) {
 // the barrier, 8 passes over the n x ld block).
 // With the Jacobi preconditioner (a.deg set) the first part also sums r.z, z = r / (deg + eps),
 // beta is the ratio of successive r.z, and p = z + beta p; the stop test stays on r.r.
+constexpr int UPD = 4;  // rows per thread whose loads the vector update keeps in flight
+
 __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   if (*(volatile int*)a.flags == 0 || *(volatile int*)(a.flags + 3) != 0) return;
   __shared__ float2 red[T * 4];
@@ -318,26 +320,42 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
                  make_float2(0.f, 0.f)};
   float2 e[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                  make_float2(0.f, 0.f)};
+  // UPD rows per thread in flight: every load of a group of rows is issued before the first
+  // use, so each thread keeps several rows' loads outstanding (HBM latency otherwise bounds the
+  // pass); the rows and the partial sums keep their order
   if (al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f) {
-    for (int64_t row = row0; row < a.n; row += rstep) {
-      const size_t i = (size_t)row * a.ld + 4 * q;
-      float4 r = *reinterpret_cast<const float4*>(a.R + i);
-      const float4 ap = *reinterpret_cast<const float4*>(a.AP + i);
-      r.x = fmaf(-al.x, ap.x, r.x);
-      r.y = fmaf(-al.y, ap.y, r.y);
-      r.z = fmaf(-al.z, ap.z, r.z);
-      r.w = fmaf(-al.w, ap.w, r.w);
-      *reinterpret_cast<float4*>(a.R + i) = r;
-      d[0] = df_fma(d[0], r.x, r.x);
-      d[1] = df_fma(d[1], r.y, r.y);
-      d[2] = df_fma(d[2], r.z, r.z);
-      d[3] = df_fma(d[3], r.w, r.w);
-      if (pc) {
-        const float4 z = f4_scale(r, jacobi_inv(a.deg, row, a.eps));
-        e[0] = df_fma(e[0], r.x, z.x);
-        e[1] = df_fma(e[1], r.y, z.y);
-        e[2] = df_fma(e[2], r.z, z.z);
-        e[3] = df_fma(e[3], r.w, z.w);
+    for (int64_t rowb = row0; rowb < a.n; rowb += UPD * rstep) {
+      float4 r[UPD], ap[UPD];
+#pragma unroll
+      for (int k = 0; k < UPD; ++k) {
+        const int64_t row = rowb + k * rstep;
+        if (row < a.n) {
+          const size_t i = (size_t)row * a.ld + 4 * q;
+          r[k] = *reinterpret_cast<const float4*>(a.R + i);
+          ap[k] = *reinterpret_cast<const float4*>(a.AP + i);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < UPD; ++k) {
+        const int64_t row = rowb + k * rstep;
+        if (row >= a.n) break;
+        float4 rr = r[k];
+        rr.x = fmaf(-al.x, ap[k].x, rr.x);
+        rr.y = fmaf(-al.y, ap[k].y, rr.y);
+        rr.z = fmaf(-al.z, ap[k].z, rr.z);
+        rr.w = fmaf(-al.w, ap[k].w, rr.w);
+        *reinterpret_cast<float4*>(a.R + (size_t)row * a.ld + 4 * q) = rr;
+        d[0] = df_fma(d[0], rr.x, rr.x);
+        d[1] = df_fma(d[1], rr.y, rr.y);
+        d[2] = df_fma(d[2], rr.z, rr.z);
+        d[3] = df_fma(d[3], rr.w, rr.w);
+        if (pc) {
+          const float4 z = f4_scale(rr, jacobi_inv(a.deg, row, a.eps));
+          e[0] = df_fma(e[0], rr.x, z.x);
+          e[1] = df_fma(e[1], rr.y, z.y);
+          e[2] = df_fma(e[2], rr.z, z.z);
+          e[3] = df_fma(e[3], rr.w, z.w);
+        }
       }
     }
   }
@@ -393,25 +411,41 @@ __global__ void __launch_bounds__(T) k_update_fused(VecArgs a) {
   const bool any_p = act.x | act.y | act.z | act.w;
   const bool any_x = al.x != 0.f || al.y != 0.f || al.z != 0.f || al.w != 0.f;
   if (!any_x && !any_p) return;
-  for (int64_t row = row0; row < a.n; row += rstep) {
-    const size_t i = (size_t)row * a.ld + 4 * q;
-    float4 p = *reinterpret_cast<const float4*>(a.P + i);
-    if (any_x) {
-      float4 x = *reinterpret_cast<const float4*>(a.X + i);
-      x.x = fmaf(al.x, p.x, x.x);
-      x.y = fmaf(al.y, p.y, x.y);
-      x.z = fmaf(al.z, p.z, x.z);
-      x.w = fmaf(al.w, p.w, x.w);
-      *reinterpret_cast<float4*>(a.X + i) = x;
+  for (int64_t rowb = row0; rowb < a.n; rowb += UPD * rstep) {
+    float4 p[UPD], x[UPD], r[UPD];
+#pragma unroll
+    for (int k = 0; k < UPD; ++k) {
+      const int64_t row = rowb + k * rstep;
+      if (row < a.n) {
+        const size_t i = (size_t)row * a.ld + 4 * q;
+        p[k] = *reinterpret_cast<const float4*>(a.P + i);
+        if (any_x) x[k] = *reinterpret_cast<const float4*>(a.X + i);
+        if (any_p) r[k] = *reinterpret_cast<const float4*>(a.R + i);
+      }
     }
-    if (!any_p) continue;
-    float4 r = *reinterpret_cast<const float4*>(a.R + i);
-    if (pc) r = f4_scale(r, jacobi_inv(a.deg, row, a.eps));  // z
-    if (act.x) p.x = fmaf(be.x, p.x, r.x);
-    if (act.y) p.y = fmaf(be.y, p.y, r.y);
-    if (act.z) p.z = fmaf(be.z, p.z, r.z);
-    if (act.w) p.w = fmaf(be.w, p.w, r.w);
-    *reinterpret_cast<float4*>(a.P + i) = p;
+#pragma unroll
+    for (int k = 0; k < UPD; ++k) {
+      const int64_t row = rowb + k * rstep;
+      if (row >= a.n) break;
+      const size_t i = (size_t)row * a.ld + 4 * q;
+      float4 pp = p[k];
+      if (any_x) {
+        float4 xx = x[k];
+        xx.x = fmaf(al.x, pp.x, xx.x);
+        xx.y = fmaf(al.y, pp.y, xx.y);
+        xx.z = fmaf(al.z, pp.z, xx.z);
+        xx.w = fmaf(al.w, pp.w, xx.w);
+        *reinterpret_cast<float4*>(a.X + i) = xx;
+      }
+      if (!any_p) continue;
+      float4 rr = r[k];
+      if (pc) rr = f4_scale(rr, jacobi_inv(a.deg, row, a.eps));  // z
+      if (act.x) pp.x = fmaf(be.x, pp.x, rr.x);
+      if (act.y) pp.y = fmaf(be.y, pp.y, rr.y);
+      if (act.z) pp.z = fmaf(be.z, pp.z, rr.z);
+      if (act.w) pp.w = fmaf(be.w, pp.w, rr.w);
+      *reinterpret_cast<float4*>(a.P + i) = pp;
+    }
   }
 }
 
