@@ -126,7 +126,9 @@ def spmm_traffic(workload):
 UPDATE_BYTES_PER_ELEM = 28
 
 
-def _traffic(kernel, workload):
+def _traffic(kernel, workload, field="dram_bytes_per_launch"):
+    """A per-launch ncu counter of `kernel` on `workload` from profiles/traffic.json, or None
+    when it was not captured or was captured on other solver sources."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
@@ -134,7 +136,7 @@ def _traffic(kernel, workload):
     e = d.get(kernel, {}).get(workload)
     if not e or e.get("solver_src_sha1") != solver_src_sha1():
         return None
-    return e.get("dram_bytes_per_launch")
+    return e.get(field)
 
 
 def solver_src_sha1():
@@ -588,6 +590,10 @@ def run_ours(args, world, rank, local_rank):
                               "rate against the HBM peak)",
                     "iterations": T, "column_iterations": float(its.sum().item()),
                     "algorithmic_bytes": algo, "launch_us": solve_us, "peak_source": src_kind}
+            l2 = None if pc else _traffic(kname[2:], args.config, "l2_bytes_per_launch")
+            if l2:  # what the solve moved through L2, by ncu's lts__t_bytes.sum
+                roof["l2_traffic"] = l2
+                roof["l2_achieved"] = l2 / (solve_us * 1e-6) / 1e9
         else:
             roof = {"bound": "hbm", "achieved": spmm["achieved"], "peak": peak, "unit": "GB/s",
                     "frac": spmm["frac"], "traffic": spmm["traffic"], "kernel": spmm["kernel"],
