@@ -162,6 +162,7 @@ def spmm_algorithmic_bytes(n, m, kc, weighted):
 # column's iteration count.
 CAPPED_EDGES = 10_000_000
 CAP_ITERS = 20
+REF_CAP_ITERS = 10  # CG iterations per step of the reference arm on such graphs
 
 
 def _oracle_solver(precond):
@@ -210,6 +211,12 @@ class OracleRun:
     def column_iterations(self, K):
         """CG iterations of column 0 solved to the tolerance (the capped samples' scale)."""
         return int(self.columns(K, 0, 1)[3][0])
+
+    def cg_only(self, Y, max_iter):
+        """(seconds, iterations) of the CG solve of the columns Y, capped at max_iter."""
+        t0 = time.perf_counter()
+        _, it, _, _ = _oracle_solver(self.precond)(self.g, self.wl.eps, Y, self.wl.tol, max_iter)
+        return time.perf_counter() - t0, int(it.max())
 
 
 def oracle_sample(run, K, cols):
@@ -321,15 +328,26 @@ def run_reference(args, world, rank):
         return
     run = OracleRun(args.config, args.precond)
     if run.capped:
-        # the iterations a column needs, from one full oracle solve (column 0), and the tail,
-        # both once; every step then times one capped column
-        T = run.column_iterations(K)
-        _, _, _, _, R = run.columns(K, 0, 1, max_iter=CAP_ITERS)
+        # once: one full oracle solve of column 0 (its right-hand side, iteration count and edge
+        # distances) and the tail; every step then times REF_CAP_ITERS CG iterations of that
+        # column and scales them to its iteration count
+        from oracle import erc_oracle as O
+
+        t_rhs, _, t_edge, it0, R = run.columns(K, 0, 1)
+        T = int(it0[0])
         t_tail = run.tail(R * K)
+        Y = O.jl_rhs(run.g, run.seed, K, 0, 1)
 
         def sample():
-            v, secs, desc, est = oracle_sample_capped(run, K, T, t_tail)
-            return v, secs, desc + f" (from a full oracle solve of column 0: {T} iterations)", est
+            t_cg, done = run.cg_only(Y, REF_CAP_ITERS)
+            est = run.t_build + K * (t_rhs + t_cg * (T / max(1, done)) + t_edge) + t_tail
+            desc = (f"full graph (n={run.n}, m={run.m}); build ({run.t_build:.1f} s), one "
+                    f"column's right-hand side ({t_rhs:.1f} s) and edge distances "
+                    f"({t_edge:.1f} s) from a full oracle solve of column 0 ({T} iterations), "
+                    f"and the curvature/probability tail ({t_tail:.1f} s) timed once; each "
+                    f"step times {done} CG iterations of that column, scaled to {T} per column "
+                    f"and to {K} columns")
+            return run.m / est, t_cg, desc, est
     else:
         cols = min(K, max(4, K // 8))
 
