@@ -196,6 +196,9 @@ def _check_run(name, n, g, prm, out, ora):
 
 
 def test_solution_residual_and_curvature_properties(big, chunk, ora):
+    """The whole run at the largest K, and the workload's smaller projections of its K sweep
+    (the 2.45M-node graph: K = 64 in one batch, K = 256 in two batches of 128), each with the
+    sampling epilogue."""
     n, g, prm, out = big["n"], big["g"], big["prm"], big["out"]
     # independent check of one batch: ||y - L_eps x|| / ||y|| through the operator kernel
     Y, X = chunk["Y"], chunk["X"]
@@ -203,22 +206,15 @@ def test_solution_residual_and_curvature_properties(big, chunk, ora):
     res = (Y - AX).double().norm(dim=0) / Y.double().norm(dim=0)
     assert float(res[:prm.kc].max()) <= 2 * prm.tol, float(res.max())
     del AX
-    ora["K"] = prm.K
+    ora["K"] = prm.K  # the oracle's columns belong to the largest projection
     _check_run(big["name"], n, g, prm, out, ora)
-
-
-@pytest.mark.parametrize("K", [64, 256])
-def test_k_sweep_of_the_large_graph(big, ora, K):
-    """The 2.45M-node workload's smaller projections (K = 64 in one batch, K = 256 in two batches
-    of 128), with the sampling epilogue."""
-    if big["name"] != "chung_lu_n2449029_g2.3":
-        pytest.skip("the K sweep belongs to the 2.45M-node workload")
     wl = big["wl"]
-    K, kc = bench_shape(wl, K)
-    prm = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
-    out = erc.erc_run(big["n"], big["src_d"], big["dst_d"], big["w_d"], prm)
-    ora["K"] = max(wl.K)  # the oracle's columns belong to the K = 1024 projection
-    _check_run(big["name"], big["n"], big["g"], prm, out, ora)
+    for Ks in sorted(set(wl.K) - {prm.K}):
+        K, kc = bench_shape(wl, Ks)
+        p2 = erc.Params(K=K, kc=kc, eps=wl.eps, tol=wl.tol, seed=synth.JL_SEED)
+        out2 = erc.erc_run(n, big["src_d"], big["dst_d"], big["w_d"], p2)
+        _check_run(big["name"], n, g, p2, out2, ora)
+        del out2
 
 
 def test_jacobi_pcg_full_size(big, chunk):
