@@ -153,6 +153,20 @@ def spmm_algorithmic_bytes(n, m, kc, weighted):
     return 4 * 2 * m + (4 * 2 * m if weighted else 0) + 8 * (n + 1) + 2 * 4 * n * kc
 
 
+def solve_algorithmic_bytes(n, m, kc, weighted, column_iters, resident):
+    """Bytes a single-launch CG solve must move: the CSR once per iteration while any column is
+    active; per column and iteration it runs, its column of P once, of Ap once and the update's
+    7 vector passes (a stopped column is neither gathered nor updated); the launch's own
+    initialisation (read Y; write P, X); and, in the resident kernel, the true residual (one
+    operator pass and Y read)."""
+    T = max(column_iters) if len(column_iters) else 0
+    csr = spmm_algorithmic_bytes(n, m, kc, weighted) - 2 * 4 * n * kc
+    algo = T * csr + sum(column_iters) * (8 + UPDATE_BYTES_PER_ELEM) * n + 12 * n * kc
+    if resident:
+        algo += spmm_algorithmic_bytes(n, m, kc, weighted) + 4 * n * kc
+    return algo
+
+
 # ------------------------------------------------------------------------------------ oracle leg
 # The float64 oracle (oracle/erc_oracle.py, as it stands) timed on the host cores on a bounded
 # sample of the workload.  A run costs build + K x (one column's right-hand side, CG solve and
@@ -593,11 +607,8 @@ def run_ours(args, world, rank, local_rank):
             # initialisation (read Y; write P, X) and, in the resident kernel, the true residual
             its = it_cg.double()
             T = int(its.max().item())
-            csr = op_bytes - 2 * 4 * n * kc
-            algo = T * csr + float(its.sum().item()) * (8 + UPDATE_BYTES_PER_ELEM) * n
-            algo += 12 * n * kc
-            if path == 1:
-                algo += op_bytes + 4 * n * kc
+            algo = solve_algorithmic_bytes(n, g.m, kc, weighted, [int(x) for x in it_cg.tolist()],
+                                           path == 1)
             ach = algo / (solve_us * 1e-6) / 1e9
             kname = "k_cg_cluster" if path == 2 else "k_cg_resident"
             roof = {"bound": "l2", "achieved": ach, "peak": peak, "unit": "GB/s",

@@ -80,3 +80,21 @@ def test_capped_oracle_sample_keeps_the_contract(monkeypatch, capsys):
     T = run.column_iterations(64)
     v, _, desc, est = bench.oracle_sample_capped(run, 64, T, cap=5)
     assert v > 0 and est > run.t_build and "5 CG iterations" in desc
+
+
+def test_solve_algorithmic_bytes():
+    """The single-launch solvers' bytes: CSR per iteration of the slowest column, 36 bytes per row
+    per column-iteration (P, Ap, 7 update passes), initialisation, and the resident kernel's
+    true-residual pass."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    n, m, kc = 1000, 5000, 4
+    iters = [10, 12, 7, 12]
+    csr = 4 * 2 * m + 8 * (n + 1)
+    expect = 12 * csr + sum(iters) * 36 * n + 12 * n * kc
+    assert bench.solve_algorithmic_bytes(n, m, kc, False, iters, False) == expect
+    assert bench.solve_algorithmic_bytes(n, m, kc, False, iters, True) == \
+        expect + bench.spmm_algorithmic_bytes(n, m, kc, False) + 4 * n * kc
+    # a weighted graph reads its CSR weights once per iteration as well
+    assert bench.solve_algorithmic_bytes(n, m, kc, True, iters, False) == expect + 12 * 4 * 2 * m
