@@ -47,12 +47,13 @@ def _solve_column(task):
     R = O.edge_resistance(g, X)
     foster = float(np.dot(np.asarray(g["ew"], dtype=np.float64), R))
     shm = shared_memory.SharedMemory(name=shm_name)
+    acc = None
     try:
         acc = np.ndarray((g["m"],), dtype=np.float64, buffer=shm.buf)
         with _lock:
             acc += R
     finally:
-        del acc
+        acc = None  # the view must go before the mapping is closed
         shm.close()
     return c, int(it[0]), float(relres[0]), bool(ok), foster
 
@@ -70,6 +71,7 @@ def oracle_columns(g, seed, K, cols, eps, tol, procs=None, precond=False):
             np.save(os.path.join(d, k + ".npy"), np.ascontiguousarray(g[k]))
         np.save(os.path.join(d, "nm.npy"), np.array([g["n"], m], dtype=np.int64))
         shm = shared_memory.SharedMemory(create=True, size=max(8, 8 * m))
+        acc = None
         try:
             acc = np.ndarray((m,), dtype=np.float64, buffer=shm.buf)
             acc[:] = 0.0
@@ -79,8 +81,8 @@ def oracle_columns(g, seed, K, cols, eps, tol, procs=None, precond=False):
             with ctx.Pool(procs, initializer=_init, initargs=(lock,)) as pool:
                 res = pool.map(_solve_column, tasks, chunksize=1)
             R = acc.copy()
-            del acc
         finally:
+            acc = None  # the view must go before the mapping is closed
             shm.close()
             shm.unlink()
     by_col = {r[0]: r for r in res}
